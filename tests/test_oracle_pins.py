@@ -1,0 +1,434 @@
+"""Pins of the CPU oracle to things other than itself (CPU only).
+
+The paper prints no worked numeric example, so every oracle function is pinned by one
+or more of: a hand-worked fixture under tests/golden/, a library routine it reduces to
+in a special case, a closed form or invariant the paper states, or brute force on tiny
+inputs.  Each pin is a ``check_*`` function of the oracle module; ``test_mutants``
+plants plausible mistakes in the oracle (on the CPU) and shows that some pin fails.
+"""
+
+import math
+
+import numpy as np
+import pytest
+import scipy.linalg
+import torch
+
+from oracle import qvla_oracle as O
+from tests.conftest import read_golden
+
+
+# --------------------------------------------------------------------------------------
+# Pins
+# --------------------------------------------------------------------------------------
+
+def check_hadamard_matches_scipy(o):
+    """Sylvester order (reading R1) is what scipy.linalg.hadamard builds."""
+    for n in [1, 2, 4, 8, 64, 512, 2048]:
+        assert np.array_equal(o.sylvester_hadamard(n), scipy.linalg.hadamard(n)), n
+
+
+def check_hadamard_orthogonal(o):
+    """H H^T = n I exactly (Sec. 4.1: normalised H is orthogonal)."""
+    for n in [2, 16, 256, 1024]:
+        h = o.sylvester_hadamard(n).astype(np.float64)
+        assert np.array_equal(h @ h.T, n * np.eye(n)), n
+
+
+def check_hadamard_golden(o):
+    g = read_golden("hadamard4.txt")
+    h4 = np.array([[int(v) for v in r] for r in g["_rows"]])
+    assert np.array_equal(o.sylvester_hadamard(4), h4)
+    assert np.allclose(o.normalized_hadamard(4), h4 / 2.0, rtol=0, atol=0)
+
+
+def check_rotate_matches_library_blockdiag(o):
+    """Block rotation = x . scipy block_diag(H_b/sqrt(b), ...) (Eq. 4 with U = I)."""
+    rng = np.random.default_rng(11)
+    for k, b in [(64, 16), (512, 512), (1024, 256), (96, 32)]:
+        x = rng.standard_normal((5, k))
+        r = scipy.linalg.block_diag(*([scipy.linalg.hadamard(b) / math.sqrt(b)] * (k // b)))
+        assert np.allclose(o.block_hadamard_rotate(x, b), x @ r, rtol=1e-12, atol=1e-12), (k, b)
+
+
+def check_rotate_linf_bound(o):
+    """The Fig. 2 caption bounds ||z H||_inf by ||z||_2 / sqrt(n).  As printed that fails
+    (z = ones gives sqrt(n) against 1); what holds is ||z H||_inf <= ||z||_1 / sqrt(n),
+    which equals ||z||_2 / sqrt(n) for a single dominant channel (one-hot z), the case
+    Sec. 4.1 describes.  Also: H preserves the 2-norm and is an involution."""
+    rng = np.random.default_rng(12)
+    for n in [8, 128, 2048]:
+        z = rng.standard_normal((20, n))
+        z[:, 3] *= 50.0
+        y = o.block_hadamard_rotate(z, n)
+        assert np.all(np.max(np.abs(y), axis=1) <= np.sum(np.abs(z), axis=1) / math.sqrt(n) * (1 + 1e-12))
+        ones = o.block_hadamard_rotate(np.ones((1, n)), n)
+        assert np.isclose(np.max(np.abs(ones)), math.sqrt(n))  # the printed 2-norm form fails here
+        assert np.allclose(np.linalg.norm(y, axis=1), np.linalg.norm(z, axis=1), rtol=1e-12)
+        assert np.allclose(o.block_hadamard_rotate(y, n), z, rtol=1e-11, atol=1e-11)
+        e = np.zeros((1, n))
+        e[0, 5] = 3.0
+        ye = o.block_hadamard_rotate(e, n)
+        assert np.allclose(np.abs(ye), 3.0 / math.sqrt(n), rtol=1e-14)
+        assert np.allclose(ye[0], 3.0 * scipy.linalg.hadamard(n)[5] / math.sqrt(n), rtol=1e-14)
+
+
+def check_rotation_invariance(o):
+    """Y = XW = (XR)(R^T W) for orthogonal R (Sec. 4.1), with R = P . BlockDiag(U_b) .
+    BlockDiag(H).  The activation side is built here from explicit matrices (a
+    permutation matrix and scipy's block_diag), independently of the oracle, so a weight
+    fold that disagrees with the upstream transform (e.g. U^T for U) fails."""
+    rng = np.random.default_rng(13)
+    k, n, m = 256, 48, 9
+    x = rng.standard_normal((m, k))
+    w = rng.standard_normal((n, k))
+    perm = rng.permutation(k)
+    rot = np.stack([np.linalg.qr(rng.standard_normal((64, 64)))[0] for _ in range(k // 64)])
+    pmat = np.eye(k)[:, perm]                      # (x P)[j] = x[perm[j]]
+    umat = scipy.linalg.block_diag(*rot)
+    x_up = x @ pmat @ umat
+    assert np.allclose(o.upstream_activation_transform(x, perm, rot, 64), x_up, rtol=1e-12, atol=1e-12)
+    for had in [64, 256]:
+        hmat = scipy.linalg.block_diag(*([scipy.linalg.hadamard(had) / math.sqrt(had)] * (k // had)))
+        xr = x_up @ hmat
+        wr = o.fold_weights(w, had, perm, rot, 64)
+        ref = x @ w.T
+        assert np.allclose(xr @ wr.T, ref, rtol=1e-11, atol=1e-11 * np.abs(ref).max())
+        assert np.allclose(wr, w @ pmat @ umat @ hmat, rtol=1e-11, atol=1e-11)
+        assert not np.allclose(xr, x)
+
+
+def check_quantizer_golden(o):
+    g = read_golden("quantizer_worked.txt")
+    z = np.array([float(v) for v in g["z"]], dtype=np.float32)
+    d = o.absmax_scale(z)
+    assert d == np.float32(g["delta"][0])
+    assert np.array_equal(o.quantize(z, d), np.array([int(v) for v in g["codes"]]))
+    ds = np.float32(g["step_delta"][0])
+    assert np.array_equal(o.quantize(z, ds), np.array([int(v) for v in g["step_codes"]]))
+
+
+def check_quantizer_bruteforce(o):
+    """Each code is the candidate in [-7, 7] nearest to z / Delta, ties to the even one
+    (Eq. 6 with reading R4), found by exhaustive search with exact float64 arithmetic."""
+    rng = np.random.default_rng(14)
+    z = (rng.standard_normal(4000) * 3).astype(np.float32)
+    # exact ties and clamped values
+    z[:40] = (np.arange(-20, 20) + 0.5).astype(np.float32) * np.float32(0.5)
+    for d in [np.float32(0.5), np.float32(0.37), np.float32(1.3)]:
+        q = o.quantize(z, d)
+        cand = np.arange(-7, 8, dtype=np.float64)
+        dist = np.abs(z.astype(np.float64)[:, None] - np.float64(d) * cand[None, :])  # exact
+        best = dist.min(axis=1, keepdims=True)
+        ok = dist == best
+        # among equally near candidates take the even one
+        choice = np.where(ok.sum(1) > 1, np.where(ok & (cand[None, :] % 2 == 0), cand[None, :], 99).min(1),
+                          cand[np.argmax(ok, axis=1)])
+        assert np.array_equal(q, choice.astype(np.int8)), d
+
+
+def check_quantizer_bounds(o):
+    """Codes lie in [-7, 7]; |z - Delta q| <= Delta/2 where no clamp applies; the
+    per-token maximum maps to +-7; an all-zero row has Delta = 0 and codes 0."""
+    rng = np.random.default_rng(15)
+    y = (rng.standard_normal((30, 256)) * rng.uniform(0.1, 10, (30, 1))).astype(np.float32)
+    y[7] = 0.0
+    q, d = o.quantize_activations_per_token(y)
+    assert q.min() >= -7 and q.max() <= 7
+    err = np.abs(y.astype(np.float64) - d.astype(np.float64)[:, None] * q)
+    assert np.all(err <= d.astype(np.float64)[:, None] / 2 * (1 + 1e-6))
+    am = np.argmax(np.abs(y), axis=1)
+    for r in range(30):
+        if r == 7:
+            assert d[r] == 0 and np.all(q[r] == 0)
+        else:
+            assert abs(int(q[r, am[r]])) == 7
+
+
+def check_pack_golden_and_roundtrip(o):
+    g = read_golden("pack_worked.txt")
+    codes = np.array([int(v) for v in g["codes"]], dtype=np.int8)
+    want = np.array([int(v, 16) for v in g["bytes"]], dtype=np.uint8)
+    assert np.array_equal(o.pack_int4(codes), want)
+    allc = np.array([[a, b] for a in range(-8, 8) for b in range(-8, 8)], dtype=np.int8).reshape(1, -1)
+    assert np.array_equal(o.unpack_int4(o.pack_int4(allc)), allc)
+
+
+def check_int_gemm_bruteforce(o):
+    """Exhaustive nested loops on tiny non-square shapes, and the +-7 extremes at K = 16384."""
+    rng = np.random.default_rng(16)
+    for m, n, k in [(3, 5, 7), (1, 8, 64), (6, 2, 33)]:
+        a = rng.integers(-8, 8, (m, k)).astype(np.int8)
+        b = rng.integers(-8, 8, (n, k)).astype(np.int8)
+        ref = np.zeros((m, n), dtype=np.int64)
+        for i in range(m):
+            for j in range(n):
+                s = 0
+                for t in range(k):
+                    s += int(a[i, t]) * int(b[j, t])
+                ref[i, j] = s
+        got = o.int_gemm(a, b)
+        assert got.shape == (m, n) and np.array_equal(got, ref), (m, n, k)
+    k = 16384
+    a = np.full((2, k), 7, np.int8)
+    a[1] = -7
+    b = np.full((3, k), 7, np.int8)
+    b[2, ::2] = -7
+    got = o.int_gemm(a, b)
+    assert np.array_equal(got, np.array([[49 * k, 49 * k, 0], [-49 * k, -49 * k, 0]]))
+
+
+def check_round_to_format(o):
+    """Single round-to-nearest-even into f16 / f32 agrees with numpy's direct float64
+    conversions; into bf16 it agrees with torch's float32 -> bfloat16 conversion."""
+    rng = np.random.default_rng(17)
+    x = np.concatenate([rng.standard_normal(20000) * 10.0 ** rng.uniform(-9, 5, 20000),
+                        [65504.0, 65519.99, 65520.0, -70000.0, 6e-8, 3e-8, 2.9e-8, 0.0, 1.0 + 2 ** -11, 1.0 + 3 * 2 ** -11]])
+    assert np.array_equal(o.round_to_format(x, "f16"), x.astype(np.float16).astype(np.float64))
+    assert np.array_equal(o.round_to_format(x, "f32"), x.astype(np.float32).astype(np.float64))
+    x32 = x.astype(np.float32)
+    tb = torch.from_numpy(x32).to(torch.bfloat16).double().numpy()
+    assert np.array_equal(o.round_to_format(x32.astype(np.float64), "bf16"), tb)
+
+
+def check_linear_golden(o):
+    """The hand-worked W4A4 linear (K = 4, H_4, two output channels)."""
+    g = read_golden("linear_worked.txt")
+    x = np.array([[float(v) for v in g["x"]]])
+    w = np.array([[float(v) for v in g["w0"]], [float(v) for v in g["w1"]]])
+    packed, wscale, wcodes = o.pack_weights(w, 4)
+    assert np.array_equal(wcodes[0], [int(v) for v in g["qw0"]])
+    assert np.array_equal(wcodes[1], [int(v) for v in g["qw1"]])
+    r = o.w4a4_linear(x, wcodes, wscale, 4, out_fmt="f16")
+    assert np.array_equal(r["qx"][0], [int(v) for v in g["qx"]])
+    assert np.array_equal(r["acc"][0], [int(v) for v in g["acc"]])
+    assert np.array_equal(r["y"][0], [float(v) for v in g["y_f16"]])
+
+
+def check_dequant_special_cases(o):
+    """Delta_x = Delta_w = 1 and no bias gives fp16(acc) exactly for |acc| <= 2048; a zero
+    activation scale gives the bias alone."""
+    acc = np.arange(-2048, 2049, dtype=np.int64).reshape(1, -1)
+    y = o.dequant_output(acc, np.ones(1, np.float32), np.ones(acc.shape[1], np.float32), None, "f16")
+    assert np.array_equal(y, acc.astype(np.float64))
+    bias = np.linspace(-3, 3, 7).astype(np.float32)
+    y = o.dequant_output(np.full((2, 7), 1234, np.int64), np.zeros(2, np.float32), np.ones(7, np.float32), bias, "f32")
+    assert np.array_equal(y, np.broadcast_to(bias.astype(np.float64), (2, 7)))
+    y = o.dequant_output(np.full((1, 7), 3, np.int64), np.full(1, 0.5, np.float32), np.full(7, 0.25, np.float32), bias, "f32")
+    assert np.allclose(y, 0.375 + bias.astype(np.float64), rtol=1e-7)
+
+
+def check_step_lookup(o):
+    """The scale of step t is table[t], exactly; t outside [0, T) is an error; per-step
+    codes are Eq. 6 with that scale."""
+    table = np.array([0.1, 0.2, 0.3, 0.4], dtype=np.float32)
+    for t in range(4):
+        assert o.step_scale_lookup(table, t) == table[t]
+    for t in (-1, 4):
+        with pytest.raises(IndexError):
+            o.step_scale_lookup(table, t)
+    y = np.linspace(-2, 2, 64, dtype=np.float32).reshape(2, 32)
+    q, d = o.quantize_activations_per_step(y, table, 2)
+    assert np.all(d == table[2])
+    assert np.array_equal(q, o.quantize(y, np.float32(table[2])))
+
+
+def check_calibration(o):
+    """A table calibrated by absmax on X_t (Eq. 6, per-tensor reading) maps the largest
+    rotated entry of X_t to +-7 and clamps nothing; q999 <= absmax; a different draw can clamp."""
+    rng = np.random.default_rng(18)
+    xs = [rng.standard_normal((16, 128)) * (1 + 0.3 * t) for t in range(4)]
+    table = o.calibrate_step_table(xs, 128)
+    assert table.dtype == np.float32 and table.shape == (4,)
+    for t, x in enumerate(xs):
+        y = o.rotate_activations(x, 128)
+        assert table[t] == np.float32(np.max(np.abs(y))) / np.float32(7)
+        q, _ = o.quantize_activations_per_step(y, table, t)
+        assert np.abs(q).max() == 7
+        assert np.count_nonzero(np.abs(y.astype(np.float64) / np.float64(table[t])) > 7.5) == 0
+    t999 = o.calibrate_step_table(xs, 128, "q999")
+    assert np.all(t999 <= table) and np.all(t999 > 0.5 * table)
+    other = [rng.standard_normal((16, 128)) * 3.0]
+    y = o.rotate_activations(other[0], 128)
+    q, _ = o.quantize_activations_per_step(y, t999, 0)
+    assert np.count_nonzero(np.abs(y / t999[0]) > 7.5) > 0 and np.abs(q).max() == 7
+
+
+def check_weight_roundtrip(o):
+    """Per-channel RTN: |W' - Delta_w q| <= Delta_w / 2 for every folded weight."""
+    rng = np.random.default_rng(19)
+    w = rng.standard_normal((40, 256)) * 0.02
+    wf = o.fold_weights(w, 64)
+    packed, scale, codes = o.pack_weights(w, 64)
+    wf32 = wf.astype(np.float32).astype(np.float64)
+    assert np.all(np.abs(wf32 - scale.astype(np.float64)[:, None] * codes) <= scale.astype(np.float64)[:, None] / 2 * (1 + 1e-6))
+    assert np.array_equal(o.unpack_int4(packed), codes)
+
+
+def check_end_to_end_band(o):
+    """Relative output error ||Y_q - XW^T||_F / ||XW^T||_F of the whole W4A4 linear lies in a
+    sane band for Gaussian data with outlier channels, and the Hadamard rotation lowers it
+    (Sec. 4.1: H spreads activation outliers; the Table 4 ablation direction)."""
+    rng = np.random.default_rng(20)
+    m, k, n = 64, 512, 256
+    x = rng.standard_normal((m, k))
+    x[:, rng.choice(k, 4, replace=False)] *= 20
+    w = rng.standard_normal((n, k)) / math.sqrt(k)
+    ref = x @ w.T
+    errs = {}
+    for had in (1, 512):
+        _, ws, wc = o.pack_weights(w, had)
+        r = o.w4a4_linear(x, wc, ws, had, out_fmt="f32")
+        errs[had] = o.relative_output_error(r["y"], ref)
+    assert 0.02 < errs[512] < 0.25, errs
+    assert errs[512] < 0.7 * errs[1], errs
+
+
+PINS = {f.__name__: f for f in [
+    check_hadamard_matches_scipy, check_hadamard_orthogonal, check_hadamard_golden,
+    check_rotate_matches_library_blockdiag, check_rotate_linf_bound, check_rotation_invariance,
+    check_quantizer_golden, check_quantizer_bruteforce, check_quantizer_bounds,
+    check_pack_golden_and_roundtrip, check_int_gemm_bruteforce, check_round_to_format,
+    check_linear_golden, check_dequant_special_cases, check_step_lookup, check_calibration,
+    check_weight_roundtrip, check_end_to_end_band,
+]}
+
+
+@pytest.mark.parametrize("name", sorted(PINS))
+def test_pin(name):
+    PINS[name](O)
+
+
+# --------------------------------------------------------------------------------------
+# Planted mistakes: each must make at least one pin fail
+# --------------------------------------------------------------------------------------
+
+def _mut_hadamard_order(n):
+    h = np.ones((1, 1), dtype=np.int64)
+    while h.shape[0] < n:
+        h = np.block([[h, -h], [h, h]])  # still orthogonal, wrong order
+    return h
+
+
+_real_rotate = O.block_hadamard_rotate
+_real_quantize = O.quantize
+_real_int_gemm = O.int_gemm
+_real_dequant = O.dequant_output
+_real_apply_block_rotation = O.apply_block_rotation
+_real_round = O.round_to_format
+
+
+def _mut_rotate_unnormalised(x, b):
+    return _real_rotate(x, b) * math.sqrt(b)
+
+
+def _mut_rot_transposed(x, rot, rot_block):
+    if rot is None:
+        return np.asarray(x, np.float64)
+    return _real_apply_block_rotation(x, np.transpose(np.asarray(rot), (0, 2, 1)), rot_block)
+
+
+def _mut_quantize_floor(z, d):
+    z64 = z.astype(np.float64)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        r = np.floor(z64 / np.float64(d) if np.ndim(d) == 0 else z64 / d.astype(np.float64))
+    return np.clip(np.nan_to_num(r), -7, 7).astype(np.int8)
+
+
+def _mut_quantize_half_away(z, d):
+    z64 = z.astype(np.float64)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        t = z64 / np.broadcast_to(np.asarray(d, np.float64), z.shape)
+    r = np.sign(t) * np.floor(np.abs(t) + 0.5)
+    return np.clip(np.nan_to_num(r), -7, 7).astype(np.int8)
+
+
+def _mut_quantize_clamp8(z, d):
+    z64 = z.astype(np.float64)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        r = np.rint(z64 / np.broadcast_to(np.asarray(d, np.float64), z.shape))
+    return np.clip(np.nan_to_num(r), -8, 8).astype(np.int8)
+
+
+def _mut_scale_by_8(z, axis=None):
+    return (np.asarray(np.max(np.abs(z), axis=axis), np.float32) / np.float32(8)).astype(np.float32)
+
+
+def _mut_pack_swapped(q):
+    u = (np.asarray(q).astype(np.int16) & 0xF).astype(np.uint8)
+    return (u[..., 1::2] | (u[..., 0::2] << 4)).astype(np.uint8)
+
+
+def _mut_unpack_no_sign(b):
+    b = np.asarray(b, np.uint8)
+    out = np.empty(b.shape[:-1] + (b.shape[-1] * 2,), dtype=np.int16)
+    out[..., 0::2] = b & 0xF
+    out[..., 1::2] = b >> 4
+    return out.astype(np.int8)
+
+
+def _mut_gemm_transposed(qx, qw):
+    return (qx.astype(np.float64) @ qw.astype(np.float64).T).T.astype(np.int64)
+
+
+def _mut_gemm_dropped_term(qx, qw):
+    return (qx[..., 1:].astype(np.float64) @ qw[..., 1:].astype(np.float64).T).astype(np.int64)
+
+
+def _mut_dequant_no_dw(acc, dx, dw, bias=None, out_fmt="f16"):
+    return _real_dequant(acc, dx, np.ones_like(np.asarray(dw)), bias, out_fmt)
+
+
+def _mut_dequant_bias_twice(acc, dx, dw, bias=None, out_fmt="f16"):
+    b2 = None if bias is None else 2 * np.asarray(bias)
+    return _real_dequant(acc, dx, dw, b2, out_fmt)
+
+
+def _mut_lookup_off_by_one(table, t):
+    table = np.asarray(table, np.float32)
+    if not (0 <= t < table.shape[0]):
+        raise IndexError(t)
+    return table[max(t - 1, 0)]
+
+
+def _mut_round_truncate(x, fmt):
+    mant, emin, emax = O._FORMATS[fmt]
+    x = np.asarray(x, np.float64)
+    out = x.copy()
+    fin = np.isfinite(x) & (x != 0)
+    _, e = np.frexp(x[fin])
+    qexp = np.maximum(e, emin + 1) - (mant + 1)
+    out[fin] = np.ldexp(np.trunc(np.ldexp(x[fin], -qexp)), qexp)
+    return out
+
+
+MUTANTS = {
+    "hadamard_wrong_order": ("sylvester_hadamard", _mut_hadamard_order),
+    "rotate_unnormalised": ("block_hadamard_rotate", _mut_rotate_unnormalised),
+    "svd_factor_transposed": ("apply_block_rotation", _mut_rot_transposed),
+    "quantize_floor": ("quantize", _mut_quantize_floor),
+    "quantize_half_away": ("quantize", _mut_quantize_half_away),
+    "quantize_clamp_8": ("quantize", _mut_quantize_clamp8),
+    "scale_divides_by_8": ("absmax_scale", _mut_scale_by_8),
+    "pack_nibbles_swapped": ("pack_int4", _mut_pack_swapped),
+    "unpack_no_sign_extension": ("unpack_int4", _mut_unpack_no_sign),
+    "gemm_transposed_output": ("int_gemm", _mut_gemm_transposed),
+    "gemm_dropped_term": ("int_gemm", _mut_gemm_dropped_term),
+    "dequant_drops_weight_scale": ("dequant_output", _mut_dequant_no_dw),
+    "dequant_bias_twice": ("dequant_output", _mut_dequant_bias_twice),
+    "step_lookup_off_by_one": ("step_scale_lookup", _mut_lookup_off_by_one),
+    "round_truncates": ("round_to_format", _mut_round_truncate),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutants(name, monkeypatch):
+    attr, fn = MUTANTS[name]
+    monkeypatch.setattr(O, attr, fn)
+    failed = []
+    for pin_name, pin in PINS.items():
+        try:
+            pin(O)
+        except Exception:  # an assertion, or the mutant breaking a shape contract
+            failed.append(pin_name)
+    assert failed, f"no pin caught the planted mistake {name}"
