@@ -1,0 +1,397 @@
+#!/usr/bin/env python
+"""Throughput of the W4A4 quantized linear hot path on the backbone-shaped gated-MLP block.
+
+One step = one pass of the whole online path over one batch: for 816 prefix tokens of hidden
+size 2048 (bf16), rotate + quantise the input (Hadamard 2048, per-token int4), the gate/up
+projection 2048 -> 2 x 16384 as one int4 GEMM whose epilogue dequantises and applies the GELU
+gate (h = gelu(gate) * up), rotate + quantise h (Hadamard 8 x 2048, per-token int4) and the
+down projection 16384 -> 2048.  Algorithmic work: 2 * 816 * (2048 * 32768 + 16384 * 2048)
+= 164.3 G integer ops per step.  Inputs are synthetic (seeded Gaussian activations with 1%
+Student-t channels, Gaussian weights) in the shapes of the Pi-0.5 backbone MLP.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Prints one JSON line (rank 0).  Under torchrun each rank runs its own replica of the block
+(weak scaling, no collective on the data path); the time is the maximum over ranks.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+M, K_IN, HIDDEN = 816, 2048, 16384
+HAD_IN, HAD_HIDDEN = 2048, 2048
+OPS_GATEUP = 2 * M * K_IN * 2 * HIDDEN
+OPS_DOWN = 2 * M * HIDDEN * K_IN
+OPS_STEP = OPS_GATEUP + OPS_DOWN
+METRIC = "W4A4 linear TOPS"
+WORKLOAD = ("backbone gated-MLP block: 816 tokens x 2048 -> gate/up 2x16384 (GELU-gated) -> down 2048, "
+            "bf16 activations, per-token int4 activations, per-channel int4 weights, Hadamard 2048")
+FP8_OVER_BF16 = 4.5 / 2.25  # nominal dense tensor-rate ratio (E4M3 operands vs bf16)
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--sets", type=int, default=3, help="rotating weight+activation sets (working set > L2)")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="CPU-baseline sample budget")
+    return ap.parse_args()
+
+
+# --------------------------------------------------------------------------------------
+# distributed plumbing (timing only; the data path has no collective)
+# --------------------------------------------------------------------------------------
+
+def dist_init():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def max_over_ranks(world, value: float, device) -> float:
+    if world == 1:
+        return value
+    import torch.distributed as dist
+
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# --------------------------------------------------------------------------------------
+# measured peaks, clocks, ncu traffic
+# --------------------------------------------------------------------------------------
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d["bf16_tflops_sustained"] * FP8_OVER_BF16, d["hbm_gbs"], "measured"
+    return 1700.0 * FP8_OVER_BF16, 6800.0, "fallback"
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.gpu = gpu_index
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = [r.split(", ") for r in out.strip().splitlines() if r.strip()]
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx = max(mx, float(r[2]))
+            except (ValueError, IndexError):
+                continue
+            for name, v in zip(names, r[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def gemm_traffic():
+    """dram bytes per launch of the GEMM kernel from the committed ncu summary, or None if the
+    kernel source changed since the counters were taken."""
+    p = os.path.join(ROOT, "profiles", "gemm_w4a4_traffic.json")
+    if not os.path.exists(p):
+        return None
+    d = json.load(open(p))
+    src = open(os.path.join(ROOT, "paper_2605_28803_gb300", "csrc", "gemm.cu"), "rb").read()
+    if hashlib.sha256(src).hexdigest() != d.get("gemm_cu_sha256"):
+        return None
+    return d.get("dram_bytes_per_step")
+
+
+# --------------------------------------------------------------------------------------
+# the workload
+# --------------------------------------------------------------------------------------
+
+def pack_workload():
+    from paper_2605_28803_gb300 import qvla as Q
+    from paper_2605_28803_gb300 import workloads as W
+
+    mlp = W.gated_mlp(seed=1, m=M, k=K_IN, hidden=HIDDEN, had_in=HAD_IN, had_hidden=HAD_HIDDEN)
+    packed = {}
+    for name, w, had in (("gate", mlp.w_gate, HAD_IN), ("up", mlp.w_up, HAD_IN), ("down", mlp.w_down, HAD_HIDDEN)):
+        n, k = w.shape
+        wq = np.zeros((n, k // 2), np.uint8)
+        ws = np.zeros(n, np.float32)
+        Q.qvla_pack_weights_host(np.ascontiguousarray(w), Q.F32, n, k, had_block=had, wq=wq, wscale=ws)
+        packed[name] = (wq, ws)
+    return mlp, packed
+
+
+def run_ours(args):
+    from paper_2605_28803_gb300 import qvla as Q
+
+    world, rank, local = dist_init()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+    mlp, packed = pack_workload()
+
+    sets = []
+    for _ in range(args.sets):
+        gu = Q.qvla_layer_create_gated(HIDDEN, K_IN, HAD_IN, Q.BF16, Q.BF16, packed["gate"][0], packed["gate"][1],
+                                       packed["up"][0], packed["up"][1])
+        dn = Q.qvla_layer_create(K_IN, HIDDEN, HAD_HIDDEN, Q.BF16, Q.BF16, packed["down"][0], packed["down"][1])
+        s = {
+            "gu": gu, "dn": dn,
+            "x": mlp.x.to(dev),
+            "xq": torch.empty(M, K_IN // 2, dtype=torch.uint8, device=dev),
+            "xs": torch.empty(M, dtype=torch.float32, device=dev),
+            "xsum": torch.empty(M, dtype=torch.int32, device=dev),
+            "h": torch.empty(M, HIDDEN, dtype=torch.bfloat16, device=dev),
+            "hq": torch.empty(M, HIDDEN // 2, dtype=torch.uint8, device=dev),
+            "hs": torch.empty(M, dtype=torch.float32, device=dev),
+            "hsum": torch.empty(M, dtype=torch.int32, device=dev),
+            "y": torch.empty(M, K_IN, dtype=torch.bfloat16, device=dev),
+        }
+        s["ws_gu"] = torch.empty(Q.qvla_linear_workspace_bytes(gu, M), dtype=torch.uint8, device=dev)
+        s["ws_dn"] = torch.empty(Q.qvla_linear_workspace_bytes(dn, M), dtype=torch.uint8, device=dev)
+        sets.append(s)
+
+    def step(s, ev=None):
+        # four launches: rotate+quantise x, gated gate/up GEMM, rotate+quantise h, down GEMM
+        Q.qvla_rotate_quantize(s["gu"], s["x"], M, -1, s["xq"], s["xs"], s["xsum"], stream)
+        if ev is not None:
+            ev[0].record(stream)
+        Q.qvla_gemm_w4a4(s["gu"], s["xq"], s["xs"], s["xsum"], M, s["h"], None, stream)
+        if ev is not None:
+            ev[1].record(stream)
+        Q.qvla_rotate_quantize(s["dn"], s["h"], M, -1, s["hq"], s["hs"], s["hsum"], stream)
+        if ev is not None:
+            ev[2].record(stream)
+        Q.qvla_gemm_w4a4(s["dn"], s["hq"], s["hs"], s["hsum"], M, s["y"], None, stream)
+        if ev is not None:
+            ev[3].record(stream)
+
+    for i in range(args.warmup):
+        step(sets[i % args.sets])
+    torch.cuda.synchronize()
+    Q.qvla_check_device(stream)
+
+    # ---- device-timed region: inputs resident in HBM ----
+    K = args.steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    t0.record(stream)
+    for i in range(K):
+        step(sets[i % args.sets], evs[i])
+    t1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop()
+    Q.qvla_check_device(stream)
+    ms = max_over_ranks(world, t0.elapsed_time(t1), dev)
+    gemm_gu_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / K
+    gemm_dn_ms = sum(e[2].elapsed_time(e[3]) for e in evs) / K
+    rq_ms = ms / K - gemm_gu_ms - gemm_dn_ms
+    value = world * OPS_STEP * K / (ms * 1e-3) / 1e12
+
+    # ---- end to end through the public API with host buffers ----
+    x_host = mlp.x.pin_memory()
+    y_host = torch.empty(M, K_IN, dtype=torch.bfloat16).pin_memory()
+    K2 = max(1, min(K, 2000))
+    barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(K2):
+        s = sets[i % args.sets]
+        s["x"].copy_(x_host, non_blocking=True)
+        Q.qvla_w4a4_linear(s["gu"], s["x"], M, -1, s["h"], s["ws_gu"], s["ws_gu"].numel(), stream)
+        Q.qvla_w4a4_linear(s["dn"], s["h"], M, -1, s["y"], s["ws_dn"], s["ws_dn"].numel(), stream)
+        y_host.copy_(s["y"], non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    Q.qvla_check_device(stream)
+    ms2 = max_over_ranks(world, e0.elapsed_time(e1), dev)
+    e2e = world * OPS_STEP * K2 / (ms2 * 1e-3) / 1e12
+
+    peak_tflops, _, peak_src = peaks()
+    achieved = (OPS_GATEUP + OPS_DOWN) / ((gemm_gu_ms + gemm_dn_ms) * 1e-3) / 1e12
+    cpu = cpu_baseline(mlp, packed, args.cpu_seconds) if (rank == 0 and world == 1) else None
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": "TOPS", "n_gpus": world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": round(ms / K, 5), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int4", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "tokens": M, "hidden": K_IN, "mlp_hidden": HIDDEN,
+                       "l2": f"{args.sets} rotating weight+activation sets (~{args.sets * 117} MB) > 129 MB L2",
+                       "parallelism": f"replica per GPU x{world}"},
+            "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": round(peak_tflops, 1),
+                         "unit": "TFLOP/s", "frac": round(achieved / peak_tflops, 4), "traffic": gemm_traffic(),
+                         "kernel": "gemm_w4a4 (gate/up + down launches)",
+                         "peak_note": f"{peak_src} sustained bf16 x {FP8_OVER_BF16:g} (nominal E4M3/bf16 ratio)"},
+            "kernels_us": {"gemm_gate_up": round(gemm_gu_ms * 1e3, 2), "gemm_down": round(gemm_dn_ms * 1e3, 2),
+                           "rotate_quantize_x_and_h": round(rq_ms * 1e3, 2)},
+            "e2e": {"value": round(e2e, 2), "unit": "TOPS", "h2d_bytes_per_step": M * K_IN * 2,
+                    "d2h_bytes_per_step": M * K_IN * 2, "steps": K2},
+            "gpu_launches": 4 * K,
+            "clocks": clk,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    for s in sets:
+        s["gu"].close()
+        s["dn"].close()
+
+
+# --------------------------------------------------------------------------------------
+# the CPU oracle (baseline leg and --impl reference)
+# --------------------------------------------------------------------------------------
+
+def oracle_block(x64, oc):
+    from oracle import qvla_oracle as O
+
+    gate = O.w4a4_linear(x64, oc["gate"][0], oc["gate"][1], HAD_IN, out_fmt="bf16")["y"]
+    up = O.w4a4_linear(x64, oc["up"][0], oc["up"][1], HAD_IN, out_fmt="bf16")["y"]
+    h = O.round_to_format(O.gated_glue(gate, up), "bf16")
+    return O.w4a4_linear(h, oc["down"][0], oc["down"][1], HAD_HIDDEN, out_fmt="bf16")["y"]
+
+
+def oracle_weights(mlp):
+    from oracle import qvla_oracle as O
+
+    out = {}
+    for name, w, had in (("gate", mlp.w_gate, HAD_IN), ("up", mlp.w_up, HAD_IN), ("down", mlp.w_down, HAD_HIDDEN)):
+        _, ws, codes = O.pack_weights(w.astype(np.float64), had)
+        out[name] = (codes, ws)
+    return out
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def cpu_baseline(mlp, packed, seconds, tokens=16):
+    """The oracle as it stands on a bounded sample: 16-token slices of the same block, repeated
+    for about `seconds` of host time.  The oracle's offline weight pack is not timed."""
+    oc = oracle_weights(mlp)
+    x64 = mlp.x.double().numpy()
+    done, t0 = 0, time.perf_counter()
+    i = 0
+    while True:
+        rows = slice((i * tokens) % M, (i * tokens) % M + tokens)
+        oracle_block(x64[rows], oc)
+        done += tokens
+        i += 1
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    ops = 2 * done * (K_IN * 2 * HIDDEN + HIDDEN * K_IN)
+    return {"value": round(ops / el / 1e12, 6), "unit": "TOPS", "cores": cpu_cores(), "kind": "oracle",
+            "sample": f"{done} tokens ({i} slices of {tokens}) of the same block, {el:.1f} s, numpy float64"}
+
+
+def run_reference(args, budget_s: float = 90.0):
+    """The oracle timed on the host, rank 0 only.  Each step is a bounded sample (4 tokens of the
+    block); the run times up to --steps steps but stops after about budget_s seconds, and
+    reports the number of steps it actually timed."""
+    world, rank, _ = dist_init()
+    if rank != 0:
+        return
+    from paper_2605_28803_gb300 import workloads as W
+
+    mlp = W.gated_mlp(seed=1, m=M, k=K_IN, hidden=HIDDEN, had_in=HAD_IN, had_hidden=HAD_HIDDEN)
+    oc = oracle_weights(mlp)
+    x64 = mlp.x.double().numpy()
+    tokens = 4
+    for i in range(min(args.warmup, 1)):
+        oracle_block(x64[:tokens], oc)
+    t0 = time.perf_counter()
+    done = 0
+    while done < args.steps:
+        r0 = (done * tokens) % M
+        oracle_block(x64[r0:r0 + tokens], oc)
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    el = time.perf_counter() - t0
+    ops = 2 * tokens * done * (K_IN * 2 * HIDDEN + HIDDEN * K_IN)
+    value = ops / el / 1e12
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TOPS", "n_gpus": world,
+        "steps": done, "warmup": min(args.warmup, 1), "ms_per_step": round(el / done * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int4", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "tokens": M, "hidden": K_IN, "mlp_hidden": HIDDEN},
+        "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": cpu_cores(), "kind": "oracle",
+                         "sample": f"{tokens} tokens of the block per step, {done} steps in {el:.1f} s "
+                                   f"(numpy float64 oracle; {args.steps} requested)"},
+        "e2e": {"value": round(value, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

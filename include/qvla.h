@@ -1,0 +1,188 @@
+/*
+ * libqvla -- the W4A4 quantized linear of Omega-QVLA (arxiv 2605.28803) on GB300 (sm_103a).
+ *
+ * The paper states the problem as Y ~= Delta_X' Delta_W' Q_X' Q_W' (Sec. 4.2, Eq. 7) after the
+ * composite rotation X' = X P R_hat, W' = P^T R_hat^T W (Sec. 4.1, Eq. 3-5), with symmetric
+ * int4 quantisation Delta = max|Z| / 7, Q = clamp(round(Z / Delta), -7, 7) (Sec. 4.2, Eq. 5-6),
+ * weight scales per output channel, activation scales per token (backbone) or from a per-step
+ * table indexed by the denoising step t (DiT head, Eq. 6 second display).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Matrices are row-major and dense.  Activations x are [M][K] (token-major), weights are
+ *    stored [N][K] (output channel n in row n, y = x W^T), outputs y are [M][N].
+ *  - Packed int4: byte j of a row holds code 2j in its low nibble and code 2j+1 in its high
+ *    nibble, each a 4-bit two's-complement integer.  The quantiser only produces [-7, 7].
+ *  - "device" pointers are CUDA global-memory addresses on the current device; "host"
+ *    pointers are ordinary CPU memory.  The caller owns every buffer it passes in; the
+ *    library owns what it allocates for a layer (packed weights, scales, bias, step table).
+ *  - Calls taking a `stream` (a cudaStream_t passed as void*, NULL = legacy default stream)
+ *    only enqueue work and return; they allocate nothing and never synchronise, so they can
+ *    be captured in a CUDA graph.  All other calls are synchronous.
+ *  - Every call returns a qvla_status.  On failure nothing was enqueued and
+ *    qvla_last_error() returns a message for the calling thread.
+ *  - Shapes: K % 128 == 0, the Hadamard block b is a power of two with 1 <= b <= 4096 and
+ *    K % b == 0 (b == 1 disables the online rotation), N % 16 == 0, 0 <= M <= 1 << 20,
+ *    K <= 16384 (so every integer accumulator is exact in float32).
+ *  - Kernels wait on nothing without a time limit.  A wait that runs out records
+ *    QVLA_ERR_TIMEOUT in a device-side word that qvla_check_device() reports.
+ */
+#ifndef QVLA_H
+#define QVLA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  QVLA_OK = 0,
+  QVLA_ERR_INVALID_ARG = 1,  /* a pointer, shape or dtype is not acceptable */
+  QVLA_ERR_UNSUPPORTED = 2,  /* well-formed but outside what the kernels implement */
+  QVLA_ERR_CUDA = 3,         /* a CUDA runtime call failed (message carries its text) */
+  QVLA_ERR_OOM = 4,          /* device or host allocation failed */
+  QVLA_ERR_STEP_RANGE = 5,   /* step t is outside [0, T) of the layer's table (or no table) */
+  QVLA_ERR_TIMEOUT = 6       /* a device-side wait ran out of its time limit */
+} qvla_status;
+
+typedef enum { QVLA_F16 = 0, QVLA_BF16 = 1, QVLA_F32 = 2 } qvla_dtype;
+
+/* Opaque device-resident layer: packed int4 weights, Delta_W, weight code sums, optional bias
+ * and optional per-step table.  Created by qvla_pack_weights / qvla_layer_create. */
+typedef struct qvla_layer qvla_layer;
+
+/* Message describing the last failure on the calling thread ("" if none).  The pointer
+ * stays valid until the next libqvla call on the same thread. */
+const char* qvla_last_error(void);
+
+/* Version of this interface; bumps on any incompatible change. */
+int qvla_abi_version(void);
+
+/* ------------------------------------------------------------------------------------------
+ * Offline weight preparation (Sec. 4.1 Eq. 4-5; Sec. 4.2 Eq. 5-6 per output channel).  Host
+ * only, touches no GPU.
+ *
+ * Folds the composite rotation into the weights, W'_n = W_n . P . BlockDiag(U_b) . BlockDiag(H_b)
+ * (the [N][K] form of W' = P^T R_hat^T W), in float64; rounds W' once to float32; then per
+ * output channel Delta_W[n] = max_k |W'[n,k]| / 7 (float32) and codes
+ * clamp(round(W'/Delta_W), -7, 7), round half to even on the exact quotient.
+ *
+ *   W         host [N][K] of dtype wdt (F16, BF16 or F32).
+ *   rot       host float64, NULL (U = I) or (K / rot_block) orthogonal blocks, each
+ *             rot_block x rot_block row-major, block b acting on channels [b*rot_block, ...).
+ *             A dense K x K factor is rot_block = K.  Orthogonality is the caller's promise.
+ *   perm      host int32 [K] or NULL: column j of W.P is column perm[j] of W (a permutation).
+ *   had_block Hadamard block b of the online rotation (the activations get the same block).
+ *   wq        host out [N][K/2] packed codes.      wscale  host out [N] Delta_W (float32).
+ *   wsum      host out [N] (may be NULL): sum over k of the weight codes of row n.
+ * ------------------------------------------------------------------------------------------ */
+qvla_status qvla_pack_weights_host(const void* W, qvla_dtype wdt, int N, int K,
+                                   const double* rot, int rot_block, const int32_t* perm,
+                                   int had_block, uint8_t* wq, float* wscale, int32_t* wsum);
+
+/* Upload already-packed weights as a layer (synchronous; allocates device memory the layer
+ * owns).  wq host [N][K/2], wscale host [N], bias host [N] float32 or NULL.  xdt is the
+ * activation dtype the layer accepts (F16, BF16 or F32); ydt the output dtype (F16 or BF16).
+ * had_block as in qvla_pack_weights_host.  *out receives the layer. */
+qvla_status qvla_layer_create(int N, int K, int had_block, qvla_dtype xdt, qvla_dtype ydt,
+                              const uint8_t* wq, const float* wscale, const float* bias,
+                              qvla_layer** out);
+
+/* A gated-MLP layer: the gate and up projections of a backbone MLP (the Pi-0.5 / PaliGemma
+ * backbone of Sec. 5.1), H output channels each, sharing one input.  They run as one GEMM whose
+ * epilogue rounds gate and up to ydt like two stand-alone linears, then writes
+ * h = ydt( gelu_tanh(gate) * up ), the input of the down projection.  The glue is the model's,
+ * not the paper's method; it is fused here only to avoid storing gate and up.
+ *   wq_gate, wq_up   host [H][K/2] packed codes (qvla_pack_weights_host of each projection)
+ *   wscale_gate/_up  host [H];  bias_gate/_up host [H] float32 or NULL.
+ * H % 128 == 0.  For this layer qvla_gemm_w4a4 and qvla_w4a4_linear write y as [M][H] (h),
+ * and the optional acc output is [M][2H]: the H gate accumulators, then the H up ones. */
+qvla_status qvla_layer_create_gated(int H, int K, int had_block, qvla_dtype xdt, qvla_dtype ydt,
+                                    const uint8_t* wq_gate, const float* wscale_gate, const uint8_t* wq_up,
+                                    const float* wscale_up, const float* bias_gate, const float* bias_up,
+                                    qvla_layer** out);
+
+/* qvla_pack_weights_host followed by qvla_layer_create (the spec entry point). */
+qvla_status qvla_pack_weights(const void* W, qvla_dtype wdt, int N, int K,
+                              const double* rot, int rot_block, const int32_t* perm,
+                              int had_block, const float* bias, qvla_dtype xdt, qvla_dtype ydt,
+                              qvla_layer** out);
+
+/* Free a layer and everything it owns (synchronises the device first).  NULL is a no-op. */
+qvla_status qvla_layer_destroy(qvla_layer* layer);
+
+/* Per-step activation scale table of Eq. 6 (second display), read as one float32 per step
+ * (per-tensor): scales host [T], each > 0 and finite, T >= 1.  Replaces any earlier table.
+ * Synchronous. */
+qvla_status qvla_set_step_scales(qvla_layer* layer, const float* scales, int T);
+
+/* Shape of a layer (N = output channels: H for a gated layer); any output pointer may be
+ * NULL.  T is 0 when no table is set. */
+qvla_status qvla_layer_info(const qvla_layer* layer, int* N, int* K, int* had_block, int* T);
+
+/* ------------------------------------------------------------------------------------------
+ * Online rotation + activation quantisation (Sec. 4.1 Eq. 5 online factor; Sec. 4.2 Eq. 5-6).
+ *
+ * For each row m of x (device [M][K], the layer's activation dtype, already in the P.U basis
+ * applied upstream): y = x_m . BlockDiag(H_b/sqrt(b)) in float32, then
+ *   step == -1 : per-token scale xscale[m] = max_k |y_k| / 7               (backbone)
+ *   step >= 0  : xscale[m] = table[step] of the layer                        (DiT, Eq. 6)
+ * and codes clamp(round(y / xscale[m]), -7, 7), round half to even on the exact quotient of
+ * the float32 operands; xscale = 0 gives codes 0.
+ *   xq      device out [M][K/2] packed codes.     xscale device out [M] float32.
+ *   xsum    device out [M] int32 (may be NULL): sum over k of the codes of row m.  The GEMM
+ *           needs it (its operand encoding is offset binary; the sum removes the offset).
+ * Returns QVLA_ERR_STEP_RANGE for step outside [0, T) (or step >= 0 without a table).
+ * ------------------------------------------------------------------------------------------ */
+qvla_status qvla_rotate_quantize(const qvla_layer* layer, const void* x, int M, int step,
+                                 uint8_t* xq, float* xscale, int32_t* xsum, void* stream);
+
+/* The same operation without a layer, for any [M][K] input of dtype xdt and any block b
+ * (b == 1: quantise x as given, no rotation).  step_scale is a DEVICE pointer to one float32
+ * used as the per-step scale, or NULL for per-token scales. */
+qvla_status qvla_rotate_quantize_rows(const void* x, qvla_dtype xdt, int M, int K, int had_block,
+                                      const float* step_scale, uint8_t* xq, float* xscale,
+                                      int32_t* xsum, void* stream);
+
+/* Calibration helper for the per-step table (Eq. 6, sigma_hat = max abs): raises the device
+ * float *absmax (which the caller initialises, e.g. to 0) to max |x . BlockDiag(H_b/sqrt(b))|
+ * over all M x K entries.  The table entry is then absmax / 7. */
+qvla_status qvla_rotated_absmax(const void* x, qvla_dtype xdt, int M, int K, int had_block,
+                                float* absmax, void* stream);
+
+/* ------------------------------------------------------------------------------------------
+ * Integer GEMM + dequantisation epilogue (Sec. 4.2 Eq. 7, scales "folded into
+ * dequantization", Sec. 5.1):
+ *   acc[m,n] = sum_k xq[m,k] * wq[n,k]                       (exact integer)
+ *   y[m,n]   = ydt( fma( (float)acc[m,n], xscale[m] * Delta_W[n], bias[n] ) )
+ * with xscale[m] * Delta_W[n] one float32 product, the fma in float32 and one
+ * round-to-nearest-even conversion to the layer's output dtype.
+ *   xq device [M][K/2], xscale device [M], xsum device [M] (from qvla_rotate_quantize),
+ *   y device out [M][N] of the layer's output dtype,
+ *   acc device out [M][N] int32, or NULL (debug/test hook: the exact integer accumulator).
+ * ------------------------------------------------------------------------------------------ */
+qvla_status qvla_gemm_w4a4(const qvla_layer* layer, const uint8_t* xq, const float* xscale,
+                           const int32_t* xsum, int M, void* y, int32_t* acc, void* stream);
+
+/* Bytes of device workspace qvla_w4a4_linear needs for M rows (a multiple of 256). */
+size_t qvla_linear_workspace_bytes(const qvla_layer* layer, int M);
+
+/* The whole online linear (Sec. 4): rotate + quantise x (as qvla_rotate_quantize, step as
+ * there), then the integer GEMM and epilogue (as qvla_gemm_w4a4).  x device [M][K], y device
+ * out [M][N].  workspace: caller-owned device memory of at least
+ * qvla_linear_workspace_bytes(layer, M) bytes, 256-byte aligned, used only during the call's
+ * kernels on `stream` (calls that overlap on the GPU must not share it). */
+qvla_status qvla_w4a4_linear(const qvla_layer* layer, const void* x, int M, int step, void* y,
+                             void* workspace, size_t workspace_bytes, void* stream);
+
+/* Synchronise `stream`, then report (and clear) the device-side error word: QVLA_OK, or
+ * QVLA_ERR_TIMEOUT if a kernel gave up waiting since the last check. */
+qvla_status qvla_check_device(void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QVLA_H */

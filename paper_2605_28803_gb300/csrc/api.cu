@@ -1,0 +1,389 @@
+// The C ABI of libqvla (include/qvla.h): argument validation, layer objects and kernel dispatch.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/qvla.h"
+#include "kernels.h"
+#include "pack.h"
+
+struct qvla_layer {
+  int N = 0, K = 0, had_block = 1, log_b = 0;  // N = weight rows (2H when gated)
+  int gated = 0;
+  int xdt = 0, ydt = 0;
+  int device = 0;
+  uint8_t* wq = nullptr;      // device [N][K/2]
+  float* wscale = nullptr;    // device [N]
+  int32_t* wsum = nullptr;    // device [N]
+  float* bias = nullptr;      // device [N] or null
+  float* table = nullptr;     // device [table_cap]
+  int T = 0, table_cap = 0;
+};
+
+namespace {
+
+thread_local std::string g_last_error;
+
+qvla_status fail(qvla_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  std::vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+qvla_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(e == cudaErrorMemoryAllocation ? QVLA_ERR_OOM : QVLA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define QVLA_CUDA(call, what)                        \
+  do {                                               \
+    cudaError_t e_ = (call);                         \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+int ilog2_exact(int v) {
+  if (v < 1 || (v & (v - 1))) return -1;
+  int l = 0;
+  while ((1 << l) < v) ++l;
+  return l;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+qvla_status check_shape(int N, int K, int had_block) {
+  if (K <= 0 || K % 128 != 0) return fail(QVLA_ERR_INVALID_ARG, "K=%d must be a positive multiple of 128", K);
+  if (K > 16384) return fail(QVLA_ERR_UNSUPPORTED, "K=%d exceeds 16384 (exact float32 accumulation bound)", K);
+  if (N <= 0 || N % 16 != 0) return fail(QVLA_ERR_INVALID_ARG, "N=%d must be a positive multiple of 16", N);
+  const int lb = ilog2_exact(had_block);
+  if (lb < 0) return fail(QVLA_ERR_INVALID_ARG, "had_block=%d is not a power of two", had_block);
+  if (had_block > 4096) return fail(QVLA_ERR_UNSUPPORTED, "had_block=%d exceeds 4096", had_block);
+  if (K % had_block != 0) return fail(QVLA_ERR_INVALID_ARG, "K=%d is not a multiple of had_block=%d", K, had_block);
+  return QVLA_OK;
+}
+
+int num_sms(int device) {
+  static std::mutex mu;
+  static std::vector<int> cache;
+  std::lock_guard<std::mutex> lk(mu);
+  if (device >= static_cast<int>(cache.size())) cache.resize(device + 1, 0);
+  if (cache[device] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, device) != cudaSuccess || v <= 0) v = 148;
+    cache[device] = v;
+  }
+  return cache[device];
+}
+
+size_t round256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+
+qvla_status check_rows(int M) {
+  if (M < 0 || M > (1 << 20)) return fail(QVLA_ERR_INVALID_ARG, "M=%d outside [0, 2^20]", M);
+  return QVLA_OK;
+}
+
+qvla_status launch_rq(const void* x, int xdt, int M, int K, int had_block, int mode, const float* step_scale,
+                      uint8_t* xq, float* xscale, int32_t* xsum, float* absmax, void* stream) {
+  qvla::RotQuantArgs a;
+  a.x = x;
+  a.xdt = xdt;
+  a.M = M;
+  a.K = K;
+  a.log_b = ilog2_exact(had_block);
+  a.inv_sqrt_b = static_cast<float>(1.0 / std::sqrt(static_cast<double>(had_block)));
+  a.mode = mode;
+  a.step_scale = step_scale;
+  a.xq = xq;
+  a.xscale = xscale;
+  a.xsum = xsum;
+  a.absmax = absmax;
+  a.stream = static_cast<cudaStream_t>(stream);
+  QVLA_CUDA(qvla::launch_rotate_quant(a), "rotate_quantize launch");
+  return QVLA_OK;
+}
+
+qvla_status resolve_step(const qvla_layer* layer, int step, const float** step_scale) {
+  if (step == -1) {
+    *step_scale = nullptr;
+    return QVLA_OK;
+  }
+  if (step < 0 || step >= layer->T)
+    return fail(QVLA_ERR_STEP_RANGE, "step %d outside the layer's table of %d steps", step, layer->T);
+  *step_scale = layer->table + step;
+  return QVLA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* qvla_last_error(void) { return g_last_error.c_str(); }
+
+int qvla_abi_version(void) { return 1; }
+
+qvla_status qvla_pack_weights_host(const void* W, qvla_dtype wdt, int N, int K, const double* rot, int rot_block,
+                                   const int32_t* perm, int had_block, uint8_t* wq, float* wscale, int32_t* wsum) {
+  g_last_error.clear();
+  if (!W || !wq || !wscale) return fail(QVLA_ERR_INVALID_ARG, "W, wq and wscale must not be NULL");
+  if (wdt != QVLA_F16 && wdt != QVLA_BF16 && wdt != QVLA_F32) return fail(QVLA_ERR_INVALID_ARG, "bad weight dtype %d", wdt);
+  if (qvla_status s = check_shape(N, K, had_block)) return s;
+  if (rot) {
+    if (rot_block <= 0 || K % rot_block != 0)
+      return fail(QVLA_ERR_INVALID_ARG, "rot_block=%d must divide K=%d", rot_block, K);
+  }
+  if (perm) {
+    std::vector<char> seen(K, 0);
+    for (int k = 0; k < K; ++k) {
+      if (perm[k] < 0 || perm[k] >= K || seen[perm[k]]) return fail(QVLA_ERR_INVALID_ARG, "perm is not a permutation of [0, K)");
+      seen[perm[k]] = 1;
+    }
+  }
+  qvla::pack_weights_host_impl(W, static_cast<int>(wdt), N, K, rot, rot_block, perm, had_block, wq, wscale, wsum);
+  return QVLA_OK;
+}
+
+static qvla_status upload_layer(int N, int K, int had_block, qvla_dtype xdt, qvla_dtype ydt, int gated,
+                                const uint8_t* wq, const float* wscale, const float* bias, qvla_layer** out) {
+  if (xdt != QVLA_F16 && xdt != QVLA_BF16 && xdt != QVLA_F32) return fail(QVLA_ERR_INVALID_ARG, "bad activation dtype %d", xdt);
+  if (ydt != QVLA_F16 && ydt != QVLA_BF16) return fail(QVLA_ERR_INVALID_ARG, "output dtype must be F16 or BF16");
+  for (int n = 0; n < N; ++n)
+    if (!(wscale[n] >= 0.0f) || std::isinf(wscale[n])) return fail(QVLA_ERR_INVALID_ARG, "wscale[%d] is not a finite non-negative float", n);
+  std::vector<int32_t> wsum(N);
+  qvla::code_sums_host(wq, N, K, wsum.data());
+  auto* L = new (std::nothrow) qvla_layer();
+  if (!L) return fail(QVLA_ERR_OOM, "host allocation failed");
+  L->gated = gated;
+  L->N = N;
+  L->K = K;
+  L->had_block = had_block;
+  L->log_b = ilog2_exact(had_block);
+  L->xdt = xdt;
+  L->ydt = ydt;
+  cudaGetDevice(&L->device);
+  const size_t wbytes = static_cast<size_t>(N) * (K / 2);
+  cudaError_t e = cudaMalloc(&L->wq, wbytes);
+  if (e == cudaSuccess) e = cudaMalloc(&L->wscale, N * sizeof(float));
+  if (e == cudaSuccess) e = cudaMalloc(&L->wsum, N * sizeof(int32_t));
+  if (e == cudaSuccess && bias) e = cudaMalloc(&L->bias, N * sizeof(float));
+  if (e == cudaSuccess) e = cudaMemcpy(L->wq, wq, wbytes, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(L->wscale, wscale, N * sizeof(float), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(L->wsum, wsum.data(), N * sizeof(int32_t), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && bias) e = cudaMemcpy(L->bias, bias, N * sizeof(float), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    qvla_layer_destroy(L);
+    return cuda_fail(e, "layer upload");
+  }
+  *out = L;
+  return QVLA_OK;
+}
+
+qvla_status qvla_layer_create(int N, int K, int had_block, qvla_dtype xdt, qvla_dtype ydt, const uint8_t* wq,
+                              const float* wscale, const float* bias, qvla_layer** out) {
+  g_last_error.clear();
+  if (!wq || !wscale || !out) return fail(QVLA_ERR_INVALID_ARG, "wq, wscale and out must not be NULL");
+  if (qvla_status s = check_shape(N, K, had_block)) return s;
+  return upload_layer(N, K, had_block, xdt, ydt, 0, wq, wscale, bias, out);
+}
+
+qvla_status qvla_layer_create_gated(int H, int K, int had_block, qvla_dtype xdt, qvla_dtype ydt, const uint8_t* wq_gate,
+                                    const float* wscale_gate, const uint8_t* wq_up, const float* wscale_up,
+                                    const float* bias_gate, const float* bias_up, qvla_layer** out) {
+  g_last_error.clear();
+  if (!wq_gate || !wscale_gate || !wq_up || !wscale_up || !out)
+    return fail(QVLA_ERR_INVALID_ARG, "weights, scales and out must not be NULL");
+  if ((bias_gate == nullptr) != (bias_up == nullptr))
+    return fail(QVLA_ERR_INVALID_ARG, "give both biases or neither");
+  if (H <= 0 || H % 128 != 0) return fail(QVLA_ERR_INVALID_ARG, "H=%d must be a positive multiple of 128", H);
+  if (qvla_status s = check_shape(2 * H, K, had_block)) return s;
+  // interleave: weight rows [256 t, 256 t + 128) = gate rows [128 t, 128 t + 128),
+  //             rows [256 t + 128, 256 t + 256) = up rows of the same hidden units
+  const size_t rb = static_cast<size_t>(K / 2);
+  std::vector<uint8_t> wq(static_cast<size_t>(2) * H * rb);
+  std::vector<float> ws(2 * H), bs(bias_gate ? 2 * H : 0);
+  for (int t = 0; t < H / 128; ++t)
+    for (int i = 0; i < 128; ++i) {
+      const int j = 128 * t + i;
+      const int rg = 256 * t + i, ru = rg + 128;
+      std::memcpy(wq.data() + rg * rb, wq_gate + j * rb, rb);
+      std::memcpy(wq.data() + ru * rb, wq_up + j * rb, rb);
+      ws[rg] = wscale_gate[j];
+      ws[ru] = wscale_up[j];
+      if (bias_gate) {
+        bs[rg] = bias_gate[j];
+        bs[ru] = bias_up[j];
+      }
+    }
+  return upload_layer(2 * H, K, had_block, xdt, ydt, 1, wq.data(), ws.data(), bias_gate ? bs.data() : nullptr, out);
+}
+
+qvla_status qvla_pack_weights(const void* W, qvla_dtype wdt, int N, int K, const double* rot, int rot_block,
+                              const int32_t* perm, int had_block, const float* bias, qvla_dtype xdt, qvla_dtype ydt,
+                              qvla_layer** out) {
+  g_last_error.clear();
+  if (qvla_status s = check_shape(N, K, had_block)) return s;
+  std::vector<uint8_t> wq;
+  std::vector<float> ws;
+  try {
+    wq.resize(static_cast<size_t>(N) * (K / 2));
+    ws.resize(N);
+  } catch (...) {
+    return fail(QVLA_ERR_OOM, "host allocation failed");
+  }
+  if (qvla_status s = qvla_pack_weights_host(W, wdt, N, K, rot, rot_block, perm, had_block, wq.data(), ws.data(), nullptr))
+    return s;
+  return qvla_layer_create(N, K, had_block, xdt, ydt, wq.data(), ws.data(), bias, out);
+}
+
+qvla_status qvla_layer_destroy(qvla_layer* L) {
+  g_last_error.clear();
+  if (!L) return QVLA_OK;
+  cudaDeviceSynchronize();
+  cudaFree(L->wq);
+  cudaFree(L->wscale);
+  cudaFree(L->wsum);
+  cudaFree(L->bias);
+  cudaFree(L->table);
+  delete L;
+  return QVLA_OK;
+}
+
+qvla_status qvla_set_step_scales(qvla_layer* L, const float* scales, int T) {
+  g_last_error.clear();
+  if (!L || !scales) return fail(QVLA_ERR_INVALID_ARG, "layer and scales must not be NULL");
+  if (T < 1 || T > (1 << 20)) return fail(QVLA_ERR_INVALID_ARG, "T=%d must be in [1, 2^20]", T);
+  for (int t = 0; t < T; ++t)
+    if (!(scales[t] > 0.0f) || std::isinf(scales[t])) return fail(QVLA_ERR_INVALID_ARG, "scales[%d] must be finite and > 0", t);
+  if (T > L->table_cap) {  // grow; a smaller or equal table is written in place (graphs keep the address)
+    QVLA_CUDA(cudaDeviceSynchronize(), "synchronise before table reallocation");
+    cudaFree(L->table);
+    L->table = nullptr;
+    L->table_cap = 0;
+    QVLA_CUDA(cudaMalloc(&L->table, T * sizeof(float)), "step table allocation");
+    L->table_cap = T;
+  }
+  QVLA_CUDA(cudaMemcpy(L->table, scales, T * sizeof(float), cudaMemcpyHostToDevice), "step table upload");
+  L->T = T;
+  return QVLA_OK;
+}
+
+qvla_status qvla_layer_info(const qvla_layer* L, int* N, int* K, int* had_block, int* T) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (N) *N = L->gated ? L->N / 2 : L->N;
+  if (K) *K = L->K;
+  if (had_block) *had_block = L->had_block;
+  if (T) *T = L->T;
+  return QVLA_OK;
+}
+
+qvla_status qvla_rotate_quantize_rows(const void* x, qvla_dtype xdt, int M, int K, int had_block, const float* step_scale,
+                                      uint8_t* xq, float* xscale, int32_t* xsum, void* stream) {
+  g_last_error.clear();
+  if (qvla_status s = check_rows(M)) return s;
+  if (qvla_status s = check_shape(16, K, had_block)) return s;
+  if (xdt != QVLA_F16 && xdt != QVLA_BF16 && xdt != QVLA_F32) return fail(QVLA_ERR_INVALID_ARG, "bad activation dtype %d", xdt);
+  if (M == 0) return QVLA_OK;
+  if (!x || !xq || !xscale) return fail(QVLA_ERR_INVALID_ARG, "x, xq and xscale must not be NULL");
+  if (!aligned16(x) || !aligned16(xq)) return fail(QVLA_ERR_INVALID_ARG, "x and xq must be 16-byte aligned");
+  return launch_rq(x, xdt, M, K, had_block, step_scale ? 1 : 0, step_scale, xq, xscale, xsum, nullptr, stream);
+}
+
+qvla_status qvla_rotate_quantize(const qvla_layer* L, const void* x, int M, int step, uint8_t* xq, float* xscale,
+                                 int32_t* xsum, void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_rows(M)) return s;
+  const float* ss = nullptr;
+  if (qvla_status s = resolve_step(L, step, &ss)) return s;
+  if (M == 0) return QVLA_OK;
+  if (!x || !xq || !xscale) return fail(QVLA_ERR_INVALID_ARG, "x, xq and xscale must not be NULL");
+  if (!aligned16(x) || !aligned16(xq)) return fail(QVLA_ERR_INVALID_ARG, "x and xq must be 16-byte aligned");
+  return launch_rq(x, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, xq, xscale, xsum, nullptr, stream);
+}
+
+qvla_status qvla_rotated_absmax(const void* x, qvla_dtype xdt, int M, int K, int had_block, float* absmax, void* stream) {
+  g_last_error.clear();
+  if (qvla_status s = check_rows(M)) return s;
+  if (qvla_status s = check_shape(16, K, had_block)) return s;
+  if (xdt != QVLA_F16 && xdt != QVLA_BF16 && xdt != QVLA_F32) return fail(QVLA_ERR_INVALID_ARG, "bad activation dtype %d", xdt);
+  if (M == 0) return QVLA_OK;
+  if (!x || !absmax) return fail(QVLA_ERR_INVALID_ARG, "x and absmax must not be NULL");
+  if (!aligned16(x)) return fail(QVLA_ERR_INVALID_ARG, "x must be 16-byte aligned");
+  return launch_rq(x, xdt, M, K, had_block, 2, nullptr, nullptr, nullptr, nullptr, absmax, stream);
+}
+
+qvla_status qvla_gemm_w4a4(const qvla_layer* L, const uint8_t* xq, const float* xscale, const int32_t* xsum, int M, void* y,
+                           int32_t* acc, void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_rows(M)) return s;
+  if (M == 0) return QVLA_OK;
+  if (!xq || !xscale || !xsum || !y) return fail(QVLA_ERR_INVALID_ARG, "xq, xscale, xsum and y must not be NULL");
+  if (!aligned16(xq) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "xq and y must be 16-byte aligned");
+  qvla::GemmArgs a;
+  a.xq = xq;
+  a.xscale = xscale;
+  a.xsum = xsum;
+  a.wq = L->wq;
+  a.wscale = L->wscale;
+  a.wsum = L->wsum;
+  a.bias = L->bias;
+  a.y = y;
+  a.ydt = L->ydt;
+  a.acc = acc;
+  a.M = M;
+  a.N = L->N;
+  a.K = L->K;
+  a.gated = L->gated;
+  a.num_sms = num_sms(L->device);
+  a.stream = static_cast<cudaStream_t>(stream);
+  QVLA_CUDA(qvla::launch_gemm_w4a4(a), "gemm launch");
+  return QVLA_OK;
+}
+
+size_t qvla_linear_workspace_bytes(const qvla_layer* L, int M) {
+  if (!L || M <= 0) return 0;
+  return round256(static_cast<size_t>(M) * (L->K / 2)) + round256(static_cast<size_t>(M) * 4) * 2;
+}
+
+qvla_status qvla_w4a4_linear(const qvla_layer* L, const void* x, int M, int step, void* y, void* workspace,
+                             size_t workspace_bytes, void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_rows(M)) return s;
+  const float* ss = nullptr;
+  if (qvla_status s = resolve_step(L, step, &ss)) return s;
+  if (M == 0) return QVLA_OK;
+  if (!x || !y || !workspace) return fail(QVLA_ERR_INVALID_ARG, "x, y and workspace must not be NULL");
+  if (!aligned16(x) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "x and y must be 16-byte aligned");
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u) return fail(QVLA_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  const size_t need = qvla_linear_workspace_bytes(L, M);
+  if (workspace_bytes < need)
+    return fail(QVLA_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed", workspace_bytes, need);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  uint8_t* xq = ws;
+  float* xscale = reinterpret_cast<float*>(ws + round256(static_cast<size_t>(M) * (L->K / 2)));
+  int32_t* xsum = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(xscale) + round256(static_cast<size_t>(M) * 4));
+  if (qvla_status s = launch_rq(x, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, xq, xscale, xsum, nullptr, stream))
+    return s;
+  return qvla_gemm_w4a4(L, xq, xscale, xsum, M, y, nullptr, stream);
+}
+
+qvla_status qvla_check_device(void* stream) {
+  g_last_error.clear();
+  unsigned int word = 0;
+  QVLA_CUDA(qvla::read_and_clear_error_word(&word, static_cast<cudaStream_t>(stream)), "device check");
+  if (word & 1u) return fail(QVLA_ERR_TIMEOUT, "a kernel wait ran out of its time limit");
+  return QVLA_OK;
+}
+
+}  // extern "C"

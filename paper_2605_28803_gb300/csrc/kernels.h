@@ -1,0 +1,51 @@
+// Host-side interface between the C ABI (api.cu) and the kernels.  Internal to libqvla.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+namespace qvla {
+
+// ---- rotate + quantise (rotate_quant.cu) ----
+struct RotQuantArgs {
+  const void* x;           // device [M][K], dtype xdt
+  int xdt;                 // 0 f16, 1 bf16, 2 f32
+  int M, K;
+  int log_b;               // log2 of the Hadamard block, 0 = none
+  float inv_sqrt_b;        // float32(1 / sqrt(b))
+  int mode;                // 0 per-token, 1 per-step (step_scale), 2 absmax only
+  const float* step_scale; // device, one float (mode 1)
+  uint8_t* xq;             // device [M][K/2]
+  float* xscale;           // device [M]
+  int32_t* xsum;           // device [M] or null
+  float* absmax;           // device, one float (mode 2)
+  cudaStream_t stream;
+};
+bool rotate_quant_supported(int log_b);
+cudaError_t launch_rotate_quant(const RotQuantArgs& a);
+
+// ---- W4A4 GEMM + epilogue (gemm.cu) ----
+struct GemmArgs {
+  const uint8_t* xq;       // device [M][K/2] activation codes
+  const float* xscale;     // device [M]
+  const int32_t* xsum;     // device [M]
+  const uint8_t* wq;       // device [N][K/2] weight codes
+  const float* wscale;     // device [N]
+  const int32_t* wsum;     // device [N]
+  const float* bias;       // device [N] or null
+  void* y;                 // device [M][N], dtype ydt
+  int ydt;                 // 0 f16, 1 bf16
+  int32_t* acc;            // device [M][N] or null
+  int M, N, K;             // N = weight rows (2H for a gated layer)
+  int gated;               // 1: rows interleave gate/up in 128-row groups; y is [M][N/2] = h
+  int num_sms;
+  cudaStream_t stream;
+};
+cudaError_t launch_gemm_w4a4(const GemmArgs& a);
+
+// Read and clear the device-side error word of the kernels that wait (gemm.cu).
+cudaError_t read_and_clear_error_word(unsigned int* out, cudaStream_t stream);
+
+}  // namespace qvla

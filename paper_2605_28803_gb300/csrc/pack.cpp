@@ -1,0 +1,161 @@
+// Offline weight preparation on the host (Sec. 4.1 Eq. 4-5 fold; Sec. 4.2 Eq. 5-6 per output
+// channel): W'_n = W_n . P . BlockDiag(U_b) . BlockDiag(H_b / sqrt(b)) in float64, rounded once
+// to float32, then Delta_W[n] = max |W'_n| / 7 (float32) and int4 codes
+// clamp(round(W'/Delta_W), -7, 7) rounded half to even on the exact quotient, nibble-packed.
+// The Hadamard factor is applied with an in-place radix-2 fast transform.
+#include "pack.h"
+
+#include <algorithm>
+#include <atomic>
+#include <cfenv>
+#include <cmath>
+#include <cstring>
+#include <thread>
+#include <vector>
+
+namespace qvla {
+namespace {
+
+float half_to_float(uint16_t h) {
+  const uint32_t sign = static_cast<uint32_t>(h & 0x8000u) << 16;
+  const uint32_t exp = (h >> 10) & 0x1Fu;
+  const uint32_t man = h & 0x3FFu;
+  uint32_t bits;
+  if (exp == 0) {
+    if (man == 0) {
+      bits = sign;
+    } else {  // subnormal: man * 2^-24
+      float f = std::ldexp(static_cast<float>(man), -24);
+      std::memcpy(&bits, &f, 4);
+      bits |= sign;
+    }
+  } else if (exp == 31) {
+    bits = sign | 0x7F800000u | (man << 13);
+  } else {
+    bits = sign | ((exp + 112u) << 23) | (man << 13);
+  }
+  float f;
+  std::memcpy(&f, &bits, 4);
+  return f;
+}
+
+float bf16_to_float(uint16_t b) {
+  const uint32_t bits = static_cast<uint32_t>(b) << 16;
+  float f;
+  std::memcpy(&f, &bits, 4);
+  return f;
+}
+
+double load_elem(const void* W, int wdt, size_t i) {
+  switch (wdt) {
+    case 0: return half_to_float(static_cast<const uint16_t*>(W)[i]);
+    case 1: return bf16_to_float(static_cast<const uint16_t*>(W)[i]);
+    default: return static_cast<const float*>(W)[i];
+  }
+}
+
+// In-place fast Walsh-Hadamard transform of n = 2^k doubles (Sylvester order), unnormalised.
+void fwht(double* v, int n) {
+  for (int h = 1; h < n; h <<= 1)
+    for (int i = 0; i < n; i += 2 * h)
+      for (int j = i; j < i + h; ++j) {
+        const double a = v[j], c = v[j + h];
+        v[j] = a + c;
+        v[j + h] = a - c;
+      }
+}
+
+// Round half to even of the exact quotient z / d for float32 z and d > 0: the float64 quotient
+// lies at least 2^-25 (relative) from any half-integer it is not equal to, so the float64
+// nearest-even rounding takes the exact decision.
+int quantize_code(float z, float d) {
+  if (!(d > 0.0f)) return 0;
+  const double t = static_cast<double>(z) / static_cast<double>(d);
+  if (std::isnan(t)) return 0;
+  double r = std::nearbyint(t);  // default rounding mode: to nearest, ties to even
+  r = std::min(7.0, std::max(-7.0, r));
+  return static_cast<int>(r);
+}
+
+void pack_row(const void* W, int wdt, int K, int n, const double* rot, int rot_block, const int32_t* perm,
+              int had_block, std::vector<double>& a, std::vector<double>& b, std::vector<float>& f, uint8_t* wq,
+              float* wscale, int32_t* wsum) {
+  const size_t base = static_cast<size_t>(n) * K;
+  for (int k = 0; k < K; ++k) a[k] = load_elem(W, wdt, base + (perm ? perm[k] : k));
+  if (rot) {
+    std::fill(b.begin(), b.end(), 0.0);
+    for (int blk = 0; blk < K / rot_block; ++blk) {
+      const double* u = rot + static_cast<size_t>(blk) * rot_block * rot_block;
+      const double* x = a.data() + static_cast<size_t>(blk) * rot_block;
+      double* o = b.data() + static_cast<size_t>(blk) * rot_block;
+      for (int i = 0; i < rot_block; ++i) {
+        const double xi = x[i];
+        if (xi == 0.0) continue;
+        const double* urow = u + static_cast<size_t>(i) * rot_block;
+        for (int j = 0; j < rot_block; ++j) o[j] += xi * urow[j];
+      }
+    }
+    a.swap(b);
+  }
+  if (had_block > 1) {
+    const double s = 1.0 / std::sqrt(static_cast<double>(had_block));
+    for (int blk = 0; blk < K / had_block; ++blk) {
+      double* v = a.data() + static_cast<size_t>(blk) * had_block;
+      fwht(v, had_block);
+      for (int i = 0; i < had_block; ++i) v[i] *= s;
+    }
+  }
+  float amax = 0.0f;
+  for (int k = 0; k < K; ++k) {
+    f[k] = static_cast<float>(a[k]);
+    amax = std::max(amax, std::fabs(f[k]));
+  }
+  const float d = amax / 7.0f;
+  wscale[n] = d;
+  int32_t sum = 0;
+  uint8_t* row = wq + static_cast<size_t>(n) * (K / 2);
+  for (int k = 0; k < K; k += 2) {
+    const int q0 = quantize_code(f[k], d), q1 = quantize_code(f[k + 1], d);
+    sum += q0 + q1;
+    row[k / 2] = static_cast<uint8_t>((q0 & 0xF) | ((q1 & 0xF) << 4));
+  }
+  if (wsum) wsum[n] = sum;
+}
+
+}  // namespace
+
+void pack_weights_host_impl(const void* W, int wdt, int N, int K, const double* rot, int rot_block,
+                            const int32_t* perm, int had_block, uint8_t* wq, float* wscale, int32_t* wsum) {
+  std::fesetround(FE_TONEAREST);
+  unsigned nt = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
+  nt = std::min<unsigned>(nt, static_cast<unsigned>(std::max(1, N)));
+  std::atomic<int> next{0};
+  auto worker = [&]() {
+    std::fesetround(FE_TONEAREST);
+    std::vector<double> a(K), b(K);
+    std::vector<float> f(K);
+    for (;;) {
+      const int n = next.fetch_add(1);
+      if (n >= N) break;
+      pack_row(W, wdt, K, n, rot, rot_block, perm, had_block, a, b, f, wq, wscale, wsum);
+    }
+  };
+  std::vector<std::thread> pool;
+  for (unsigned i = 1; i < nt; ++i) pool.emplace_back(worker);
+  worker();
+  for (auto& t : pool) t.join();
+}
+
+void code_sums_host(const uint8_t* wq, int N, int K, int32_t* wsum) {
+  for (int n = 0; n < N; ++n) {
+    const uint8_t* row = wq + static_cast<size_t>(n) * (K / 2);
+    int32_t s = 0;
+    for (int j = 0; j < K / 2; ++j) {
+      int lo = row[j] & 0xF, hi = row[j] >> 4;
+      s += (lo >= 8 ? lo - 16 : lo) + (hi >= 8 ? hi - 16 : hi);
+    }
+    wsum[n] = s;
+  }
+}
+
+}  // namespace qvla

@@ -1,0 +1,115 @@
+"""CPU tests of the C ABI: the library loads, exports every symbol include/qvla.h declares,
+rejects bad arguments before touching a GPU, and its host-only weight pack (fold + per-channel
+int4 RTN + nibble packing) matches the oracle bit for bit."""
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import qvla_oracle as O
+from paper_2605_28803_gb300 import qvla as Q
+from paper_2605_28803_gb300 import workloads as W
+from tests.conftest import ROOT
+
+
+def header_symbols():
+    src = open(os.path.join(ROOT, "include", "qvla.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(qvla_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported():
+    names = header_symbols()
+    assert len(names) >= 15
+    lib = ctypes.CDLL(Q._LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+    assert sorted(Q.SIGNATURES) == names
+
+
+def test_abi_version():
+    assert Q.qvla_abi_version() == 1
+
+
+@pytest.mark.parametrize("N,K,had", [(16, 100, 4), (15, 128, 128), (16, 128, 3), (16, 128, 256), (16, 32768, 1024),
+                                     (16, 256, 8192)])
+def test_pack_rejects_bad_shapes(N, K, had):
+    w = np.zeros((max(N, 1), K), np.float32)
+    wq = np.zeros((max(N, 1), K // 2), np.uint8)
+    ws = np.zeros(max(N, 1), np.float32)
+    with pytest.raises(Q.QvlaError) as e:
+        Q.qvla_pack_weights_host(w, Q.F32, N, K, had_block=had, wq=wq, wscale=ws)
+    assert e.value.status in (1, 2)
+
+
+def test_pack_rejects_bad_permutation():
+    N, K = 16, 128
+    w = np.zeros((N, K), np.float32)
+    perm = np.arange(K, dtype=np.int32)
+    perm[3] = 5
+    with pytest.raises(Q.QvlaError):
+        Q.qvla_pack_weights_host(w, Q.F32, N, K, perm=perm, had_block=128, wq=np.zeros((N, K // 2), np.uint8),
+                                 wscale=np.zeros(N, np.float32))
+
+
+def test_validation_precedes_any_device_work():
+    # bad K / dtype / step are reported without a GPU; M = 0 is a no-op
+    with pytest.raises(Q.QvlaError) as e:
+        Q.qvla_rotate_quantize_rows(None, Q.F16, 4, 100, 1, None, None, None)
+    assert e.value.status == 1
+    with pytest.raises(Q.QvlaError):
+        Q.qvla_rotate_quantize_rows(None, 7, 4, 128, 1, None, None, None)
+    Q.qvla_rotate_quantize_rows(None, Q.F16, 0, 128, 1, None, None, None)
+    with pytest.raises(Q.QvlaError):
+        Q.qvla_rotated_absmax(None, Q.F16, 1 << 21, 128, 1, None)
+
+
+def _host_pack(w, wdt, had, rot=None, rot_block=0, perm=None):
+    N, K = w.shape
+    wq = np.zeros((N, K // 2), np.uint8)
+    ws = np.zeros(N, np.float32)
+    wsum = np.zeros(N, np.int32)
+    Q.qvla_pack_weights_host(np.ascontiguousarray(w), wdt, N, K, rot=rot, rot_block=rot_block, perm=perm,
+                             had_block=had, wq=wq, wscale=ws, wsum=wsum)
+    return wq, ws, wsum
+
+
+@pytest.mark.parametrize("dtype", ["f16", "bf16", "f32"])
+@pytest.mark.parametrize("N,K,had", [(48, 512, 512), (32, 2048, 2048), (16, 1024, 64), (16, 256, 1)])
+def test_host_pack_matches_oracle(dtype, N, K, had):
+    rng = np.random.default_rng(N * K + had)
+    w = W.gaussian_weights(rng, N, K, 0.02)
+    w[:, 3] *= 30
+    wt = W.as_dtype(w, dtype)
+    raw = wt.view(torch.int16).numpy() if dtype != "f32" else wt.numpy()
+    wq, ws, wsum = _host_pack(raw, Q.DTYPE_CODES[dtype], had)
+    oq, osc, oc = O.pack_weights(wt.double().numpy(), had)
+    assert np.array_equal(ws, osc)
+    assert np.array_equal(wq, oq)
+    assert np.array_equal(wsum, oc.astype(np.int64).sum(1))
+
+
+def test_host_pack_with_svd_factor_and_permutation_matches_oracle():
+    rng = np.random.default_rng(5)
+    N, K = 64, 512
+    w = W.gaussian_weights(rng, N, K, 0.02)
+    perm = rng.permutation(K).astype(np.int32)
+    rot = np.stack([W.random_orthogonal(rng, 128) for _ in range(K // 128)])
+    wq, ws, _ = _host_pack(w, Q.F32, 256, rot=np.ascontiguousarray(rot), rot_block=128, perm=perm)
+    oq, osc, oc = O.pack_weights(w.astype(np.float64), 256, perm=perm, rot=rot, rot_block=128)
+    # the fold is float64 on both sides but in a different order (fast transform vs dense
+    # product); codes may only differ where a float64 rounding crosses a float32 boundary
+    assert np.array_equal(ws, osc)
+    diff = np.count_nonzero(O.unpack_int4(wq) != oc)
+    assert diff == 0
+
+
+def test_host_pack_dense_svd_factor_config1():
+    case = W.single_layer_steps(seed=0)
+    wq, ws, _ = _host_pack(case.w, Q.F32, case.had_block, rot=np.ascontiguousarray(case.rot), rot_block=case.rot_block)
+    oq, osc, _ = O.pack_weights(case.w.astype(np.float64), case.had_block, rot=case.rot, rot_block=case.rot_block)
+    assert np.array_equal(ws, osc) and np.array_equal(wq, oq)
