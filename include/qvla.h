@@ -177,6 +177,29 @@ size_t qvla_linear_workspace_bytes(const qvla_layer* layer, int M);
 qvla_status qvla_w4a4_linear(const qvla_layer* layer, const void* x, int M, int step, void* y,
                              void* workspace, size_t workspace_bytes, void* stream);
 
+/* Allocation-free variant of qvla_w4a4_linear.  The paper has no counterpart: this entry
+ * point exists for callers that must not allocate device memory once they are running --
+ * for example a robot controller's real-time loop, which reserves all of its memory at start-up
+ * because an allocation inside the loop can stall for milliseconds or fail mid-episode, or a
+ * plug-in whose host runtime hands out device memory only from its own pool.  Such a caller
+ * cannot provide qvla_w4a4_linear's workspace on demand, so this call uses a fixed scratch area
+ * that the library itself holds instead.
+ *
+ * The scratch is one file-scope device array of QVLA_NOALLOC_SCRATCH_BYTES (8 MiB).  Every GPU
+ * that loads the library holds it until the process exits.  The call allocates nothing: it
+ * makes no cudaMalloc/cudaFree and calls no allocating library routine.  Its first call on each
+ * device looks up the array's device address with that device current; make that first call
+ * before any stream capture.  The scratch must hold qvla_linear_workspace_bytes(layer, M)
+ * bytes (the codes [M][K/2], scales and code sums); larger requests fail with
+ * QVLA_ERR_UNSUPPORTED and enqueue nothing.  Every call shares the one array and leaves the
+ * last call's contents in it; each call overwrites all it reads, so nothing needs clearing
+ * in between.  Two calls whose kernels overlap on the GPU (different streams or threads, on
+ * the same device) race on the array: issue them on one stream.
+ * Arguments and results are those of qvla_w4a4_linear without the workspace. */
+#define QVLA_NOALLOC_SCRATCH_BYTES ((size_t)8 << 20)
+qvla_status qvla_w4a4_linear_noalloc(const qvla_layer* layer, const void* x, int M, int step, void* y,
+                                     void* stream);
+
 /* Synchronise `stream`, then report (and clear) the device-side error word: QVLA_OK, or
  * QVLA_ERR_TIMEOUT if a kernel gave up waiting since the last check. */
 qvla_status qvla_check_device(void* stream);

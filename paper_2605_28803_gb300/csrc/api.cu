@@ -378,6 +378,47 @@ qvla_status qvla_w4a4_linear(const qvla_layer* L, const void* x, int M, int step
   return qvla_gemm_w4a4(L, xq, xscale, xsum, M, y, nullptr, stream);
 }
 
+}  // extern "C"
+
+// ---- allocation-free linear: a fixed scratch area in this translation unit ----
+namespace {
+static __device__ __align__(256) uint8_t g_noalloc_scratch[QVLA_NOALLOC_SCRATCH_BYTES];
+std::mutex g_noalloc_mu;
+std::vector<void*> g_noalloc_addr;  // device address of g_noalloc_scratch, per device
+
+// The array's name in host code is only a host-side stand-in; its device address comes from
+// cudaGetSymbolAddress, looked up once per device with that device current.
+qvla_status noalloc_scratch(void** out) {
+  int dev = 0;
+  QVLA_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (dev >= static_cast<int>(g_noalloc_addr.size())) g_noalloc_addr.resize(dev + 1, nullptr);
+  if (g_noalloc_addr[dev] == nullptr) {
+    void* p = nullptr;
+    QVLA_CUDA(cudaGetSymbolAddress(&p, g_noalloc_scratch), "cudaGetSymbolAddress of the no-alloc scratch");
+    g_noalloc_addr[dev] = p;
+  }
+  *out = g_noalloc_addr[dev];
+  return QVLA_OK;
+}
+}  // namespace
+
+extern "C" {
+
+qvla_status qvla_w4a4_linear_noalloc(const qvla_layer* L, const void* x, int M, int step, void* y, void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_rows(M)) return s;
+  const size_t need = qvla_linear_workspace_bytes(L, M);
+  if (need > QVLA_NOALLOC_SCRATCH_BYTES)
+    return fail(QVLA_ERR_UNSUPPORTED, "M=%d, K=%d needs %zu bytes of scratch; the allocation-free linear holds %zu", M, L->K,
+                need, static_cast<size_t>(QVLA_NOALLOC_SCRATCH_BYTES));
+  if (M == 0) return qvla_w4a4_linear(L, x, M, step, y, nullptr, 0, stream);
+  void* scratch = nullptr;
+  if (qvla_status s = noalloc_scratch(&scratch)) return s;
+  return qvla_w4a4_linear(L, x, M, step, y, scratch, QVLA_NOALLOC_SCRATCH_BYTES, stream);
+}
+
 qvla_status qvla_check_device(void* stream) {
   g_last_error.clear();
   unsigned int word = 0;

@@ -39,6 +39,7 @@ SIGNATURES = {
     "qvla_gemm_w4a4": (_I, [_P, _P, _P, _P, _I, _P, _P, _P]),
     "qvla_linear_workspace_bytes": (_S, [_P, _I]),
     "qvla_w4a4_linear": (_I, [_P, _P, _I, _I, _P, _P, _S, _P]),
+    "qvla_w4a4_linear_noalloc": (_I, [_P, _P, _I, _I, _P, _P]),
     "qvla_check_device": (_I, [_P]),
 }
 
@@ -184,6 +185,15 @@ def qvla_linear_workspace_bytes(layer: Layer, M: int) -> int:
 def qvla_w4a4_linear(layer: Layer, x, M: int, step: int, y, workspace, workspace_bytes: int, stream=None) -> None:
     _check(_lib.qvla_w4a4_linear(layer.handle, _ptr(x), M, step, _ptr(y), _ptr(workspace), workspace_bytes,
                                  _stream(stream)))
+
+
+NOALLOC_SCRATCH_BYTES = 8 << 20
+
+
+def qvla_w4a4_linear_noalloc(layer: Layer, x, M: int, step: int, y, stream=None) -> None:
+    """qvla_w4a4_linear without a caller workspace: for callers that cannot allocate device
+    memory while running; the library's fixed 8 MiB scratch takes the workspace's place."""
+    _check(_lib.qvla_w4a4_linear_noalloc(layer.handle, _ptr(x), M, step, _ptr(y), _stream(stream)))
 
 
 def qvla_check_device(stream=None) -> None:
