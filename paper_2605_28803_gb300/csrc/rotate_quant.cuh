@@ -1,0 +1,368 @@
+// Fused online rotation + symmetric int4 activation quantisation (Sec. 4.1 Eq. 3-5, the online
+// block-Hadamard factor; Sec. 4.2 Eq. 5-6 with per-token or per-step scales).
+//
+// One row of x is spread over K/EPT threads, EPT consecutive elements each (16-byte loads),
+// held as float2 pairs.  The fast Walsh-Hadamard transform of a block of b = 2^LOGB elements
+// runs its butterfly stages on the low log2(EPT) index bits in registers (stages of distance
+// >= 2 as packed f32x2 adds/subs), then transposes once through shared memory so that each
+// thread holds the elements that differ in the remaining bits, and runs those in registers
+// too.  The scale (per token: max |y| / 7; or the step's table entry), the int4 codes, their
+// packing and the row's code sum follow from registers.  Instantiated per input dtype in
+// rotate_quant_{f16,bf16,f32}.cu.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "kernels.h"
+
+namespace qvla {
+namespace rq {
+
+constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23: t + kMagic rounds |t| < 2^22 to an integer, half to even
+// The fast path t = y * (c / delta) is within 2^-20 of the exact z / delta (|t| <= 8); a value
+// closer than this to a half-integer is decided exactly instead.
+constexpr float kTieBand = 0.5f - 7.62939453125e-6f;  // 0.5 - 2^-17
+
+template <typename T>
+struct Loader;
+
+template <>
+struct Loader<__half> {
+  static constexpr int kPer16B = 8;
+  __device__ __forceinline__ static void load(const void* p, float2* v) {
+    uint4 u = __ldg(reinterpret_cast<const uint4*>(p));
+    const __half2* h = reinterpret_cast<const __half2*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) v[i] = __half22float2(h[i]);
+  }
+};
+
+template <>
+struct Loader<__nv_bfloat16> {
+  static constexpr int kPer16B = 8;
+  __device__ __forceinline__ static void load(const void* p, float2* v) {
+    uint4 u = __ldg(reinterpret_cast<const uint4*>(p));
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) v[i] = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u));
+  }
+};
+
+template <>
+struct Loader<float> {
+  static constexpr int kPer16B = 4;
+  __device__ __forceinline__ static void load(const void* p, float2* v) {
+    float4 f = __ldg(reinterpret_cast<const float4*>(p));
+    v[0] = make_float2(f.x, f.y);
+    v[1] = make_float2(f.z, f.w);
+  }
+};
+
+__device__ __forceinline__ void bfly2(float2& a, float2& c) {  // (a, c) -> (a + c, a - c), two lanes at once
+  float2 s, d;
+  asm("{\n.reg .b64 ra, rc, rs, rd;\n"
+      "mov.b64 ra, {%4, %5};\nmov.b64 rc, {%6, %7};\n"
+      "add.rn.f32x2 rs, ra, rc;\nsub.rn.f32x2 rd, ra, rc;\n"
+      "mov.b64 {%0, %1}, rs;\nmov.b64 {%2, %3}, rd;\n}\n"
+      : "=f"(s.x), "=f"(s.y), "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(c.x), "f"(c.y));
+  a = s;
+  c = d;
+}
+
+// Butterflies on element-index bits [lo, hi) of v (kN float2 = 2 kN elements; bit 0 is the
+// pair's own lane).
+template <int kN, int kLo, int kHi>
+__device__ __forceinline__ void fwht_regs(float2 (&v)[kN]) {
+  if constexpr (kLo == 0 && kHi > 0) {
+#pragma unroll
+    for (int i = 0; i < kN; ++i) {
+      const float a = v[i].x, c = v[i].y;
+      v[i] = make_float2(a + c, a - c);
+    }
+  }
+#pragma unroll
+  for (int bit = (kLo > 1 ? kLo : 1); bit < kHi; ++bit) {
+    const int h = 1 << (bit - 1);  // distance in float2 units
+#pragma unroll
+    for (int i = 0; i < kN; ++i)
+      if ((i & h) == 0) bfly2(v[i], v[i + h]);
+  }
+}
+
+// The exact decision for one value (rare: only within 2^-17 of a tie, or when 1/delta
+// overflows): round half to even of the exact quotient z / delta for z = float32(y * c), by
+// the sign of z - h delta (one FMA is exact in sign) at the half-integer h next to t, then the
+// clamp.  Returns kMagic + q.
+static __device__ __noinline__ float exact_code(float y, float c, float delta, float cr) {
+  const float z = y * c;
+  if (isinf(cr)) return fminf(fmaxf(__fdiv_rn(z, delta), -7.0f), 7.0f) + kMagic;  // tiny delta
+  const float t = fminf(fmaxf(y * cr, -7.0f), 7.0f);
+  if (fabsf(t - ((t + kMagic) - kMagic)) < kTieBand) return t + kMagic;  // not near a tie
+  const float fl = floorf(t);
+  const float d = fmaf(-(fl + 0.5f), delta, z);
+  float q = d > 0.0f ? fl + 1.0f : fl;
+  if (d == 0.0f) q = (static_cast<int>(fl) & 1) ? fl + 1.0f : fl;
+  q = fminf(fmaxf(q, -7.0f), 7.0f);
+  return q + kMagic;
+}
+
+// 8 codes (as kMagic + q floats) -> one packed word, code 2j in the low nibble of byte j.
+__device__ __forceinline__ uint32_t pack8(const float (&u)[8]) {
+  uint32_t b[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const uint32_t lo = __float_as_uint(u[2 * j]), hi = __float_as_uint(u[2 * j + 1]) << 4;
+    b[j] = (lo & 0x0Fu) | (hi & 0xF0u);
+  }
+  return __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
+}
+
+// Sum of the 8 two's-complement codes of a packed word, plus 64 (each code offset by 8).
+__device__ __forceinline__ uint32_t sum8_offset(uint32_t w, uint32_t acc) {
+  const uint32_t o = w ^ 0x88888888u;
+  const uint32_t s = (o & 0x0F0F0F0Fu) + ((o >> 4) & 0x0F0F0F0Fu);
+  return __dp4a(s, 0x01010101u, acc);
+}
+
+// kLogB: log2 of the Hadamard block (0 = no rotation).  kEpt: elements per thread.
+// kStep: the scale is the step table entry (else per token; per-token mode also serves the
+// calibration max when absmax_out is set).
+template <typename T, int kLogB, int kEpt, bool kStep>
+__global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__ x, int M, int K, float inv_sqrt_b,
+                                                             const float* __restrict__ step_scale,
+                                                             uint8_t* __restrict__ xq, float* __restrict__ xscale,
+                                                             int32_t* __restrict__ xsum, float* __restrict__ absmax_out) {
+  constexpr int kP = (kEpt == 128) ? 7 : 6;  // log2(kEpt)
+  static_assert((1 << kP) == kEpt, "EPT");
+  constexpr int kN = kEpt / 2;                // float2 per thread
+  constexpr bool kPhase2 = kLogB > kP;
+  constexpr int kR = kPhase2 ? kLogB - kP : 0;  // bits handled after the transpose
+  constexpr int kL = kP - kR;                  // contiguous low bits per run after the transpose
+  static_assert(!kPhase2 || kL >= 1, "every run must hold whole nibble pairs");
+  constexpr int kRun = kPhase2 ? (1 << kL) : kEpt;  // contiguous elements per run
+  constexpr int kNV = kEpt / 4;                     // float4 per shared-memory line
+
+  extern __shared__ float4 smem4[];
+  __shared__ unsigned int s_max[32];
+  __shared__ unsigned int s_sum[32];
+
+  const int tpr = K / kEpt;           // threads per row
+  const int rpc = blockDim.x / tpr;   // rows per CTA
+  const int tid = threadIdx.x;
+  const int rloc = tid / tpr;         // row within the CTA
+  const int j = tid - rloc * tpr;     // thread within the row
+  const int m = blockIdx.x * rpc + rloc;
+  const bool active = (rloc < rpc) && (m < M);
+
+  if (tid < 32) {
+    s_max[tid] = 0u;
+    s_sum[tid] = 0u;
+  }
+
+  float2 v[kN];
+  if (active) {
+    const T* src = x + static_cast<size_t>(m) * K + static_cast<size_t>(j) * kEpt;
+#pragma unroll
+    for (int c = 0; c < kEpt / Loader<T>::kPer16B; ++c)
+      Loader<T>::load(src + c * Loader<T>::kPer16B, v + c * (Loader<T>::kPer16B / 2));
+  } else {
+#pragma unroll
+    for (int i = 0; i < kN; ++i) v[i] = make_float2(0.0f, 0.0f);
+  }
+  __syncthreads();
+
+  constexpr int kLowBits = kLogB < kP ? kLogB : kP;
+  fwht_regs<kN, 0, kLowBits>(v);
+
+  if constexpr (kPhase2) {
+    float4* s4 = reinterpret_cast<float4*>(reinterpret_cast<float*>(smem4) + static_cast<size_t>(rloc) * K);
+#pragma unroll
+    for (int c = 0; c < kNV; ++c) {
+      const int line = j;
+      s4[line * kNV + (c ^ (line & (kNV - 1)))] = make_float4(v[2 * c].x, v[2 * c].y, v[2 * c + 1].x, v[2 * c + 1].y);
+    }
+    __syncthreads();
+    const int jlo = j & ((1 << kR) - 1);
+    const int jhi = j >> kR;
+#pragma unroll
+    for (int ih = 0; ih < (1 << kR); ++ih) {
+      const int line = (jhi << kR) | ih;
+      const int col = jlo << kL;
+      if constexpr (kL >= 2) {
+#pragma unroll
+        for (int c = 0; c < (1 << (kL - 2)); ++c) {
+          const int vv = (col >> 2) + c;
+          const float4 f = s4[line * kNV + (vv ^ (line & (kNV - 1)))];
+          const int r = ((ih << kL) + 4 * c) >> 1;
+          v[r] = make_float2(f.x, f.y);
+          v[r + 1] = make_float2(f.z, f.w);
+        }
+      } else {  // kL == 1: one pair
+        const int vv = col >> 2;
+        v[ih] = *reinterpret_cast<const float2*>(
+            reinterpret_cast<const float*>(s4 + line * kNV + (vv ^ (line & (kNV - 1)))) + (col & 3));
+      }
+    }
+    fwht_regs<kN, kL, kP>(v);
+  }
+
+  // ---- scale ----
+  float delta;
+  if constexpr (kStep) {
+    delta = __ldg(step_scale);
+  } else {
+    float w = 0.0f;
+#pragma unroll
+    for (int i = 0; i < kN; ++i) w = fmaxf(w, fmaxf(fabsf(v[i].x), fabsf(v[i].y)));
+    if ((tpr & 31) == 0) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) w = fmaxf(w, __shfl_xor_sync(0xffffffffu, w, o));
+      if ((tid & 31) == 0) atomicMax(&s_max[rloc], __float_as_uint(w));
+    } else if ((tpr & (tpr - 1)) == 0) {
+      for (int o = tpr >> 1; o > 0; o >>= 1) w = fmaxf(w, __shfl_xor_sync(0xffffffffu, w, o));
+      if (j == 0) atomicMax(&s_max[rloc], __float_as_uint(w));
+    } else {
+      atomicMax(&s_max[rloc], __float_as_uint(w));
+    }
+    __syncthreads();
+    // max |Z| of the normalised rotation: rounding is monotone, so round(max * c) = max round(y * c)
+    const float zmax = __uint_as_float(s_max[rloc]) * inv_sqrt_b;
+    if (absmax_out != nullptr) {  // calibration: one atomic per row
+      if (active && j == 0) atomicMax(reinterpret_cast<unsigned int*>(absmax_out), __float_as_uint(zmax));
+      return;
+    }
+    delta = __fdiv_rn(zmax, 7.0f);
+  }
+  if (active && j == 0) xscale[m] = delta;
+
+  // ---- codes ----
+  const bool zero_scale = !(delta > 0.0f);
+  const float rcp = zero_scale ? 0.0f : __fdiv_rn(1.0f, delta);
+  const bool tiny_scale = !zero_scale && isinf(rcp);  // 1/delta overflows: plain division
+  const float cr = inv_sqrt_b * rcp;                  // y * cr ~ z / delta (0 when delta = 0: codes 0)
+  // codes in register order, 8 per word (register element r = 8 g + i)
+  uint32_t pk[kEpt / 8];
+  uint32_t sum_acc = 0;
+#pragma unroll
+  for (int g = 0; g < kEpt / 8; ++g) {
+    float u[8];
+    bool tie = false;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int idx = 8 * g + i;
+      const float y = (idx & 1) ? v[idx >> 1].y : v[idx >> 1].x;
+      float t = y * cr;
+      if constexpr (kStep) t = fminf(fmaxf(t, -7.0f), 7.0f);
+      u[i] = t + kMagic;
+      tie |= fabsf(t - (u[i] - kMagic)) >= kTieBand;
+    }
+    if (tie || tiny_scale) {  // rare: decide these values exactly
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int idx = 8 * g + i;
+        u[i] = exact_code((idx & 1) ? v[idx >> 1].y : v[idx >> 1].x, inv_sqrt_b, delta, cr);
+      }
+    }
+    pk[g] = pack8(u);
+    sum_acc = sum8_offset(pk[g], sum_acc);
+  }
+
+  // ---- store: run r holds register elements [r kRun, (r + 1) kRun), contiguous in the row ----
+  if (active) {
+    uint8_t* dst = xq + static_cast<size_t>(m) * (K / 2);
+#pragma unroll
+    for (int run = 0; run < kEpt / kRun; ++run) {
+      int e0;  // first element of this run within the row
+      if constexpr (kPhase2) {
+        e0 = ((j >> kR) << kLogB) | (run << kP) | ((j & ((1 << kR) - 1)) << kL);
+      } else {
+        e0 = j * kEpt;
+      }
+      uint8_t* p = dst + (e0 >> 1);
+      constexpr int kBytes = kRun / 2;
+      const int b0 = run * kBytes;  // first byte of the run in pk
+      if constexpr (kBytes == 1) {
+        *p = static_cast<uint8_t>(pk[b0 >> 2] >> (8 * (b0 & 3)));
+      } else if constexpr (kBytes == 2) {
+        *reinterpret_cast<uint16_t*>(p) = static_cast<uint16_t>(pk[b0 >> 2] >> (8 * (b0 & 3)));
+      } else if constexpr (kBytes == 4) {
+        *reinterpret_cast<uint32_t*>(p) = pk[b0 >> 2];
+      } else if constexpr (kBytes == 8) {
+        *reinterpret_cast<uint2*>(p) = make_uint2(pk[b0 >> 2], pk[(b0 >> 2) + 1]);
+      } else {
+#pragma unroll
+        for (int w = 0; w < kBytes / 4; w += 4)
+          *reinterpret_cast<uint4*>(p + 4 * w) =
+              make_uint4(pk[(b0 >> 2) + w], pk[(b0 >> 2) + w + 1], pk[(b0 >> 2) + w + 2], pk[(b0 >> 2) + w + 3]);
+      }
+    }
+  }
+  if (xsum != nullptr) {
+    int cs = static_cast<int>(sum_acc) - 8 * kEpt;  // every code carried an offset of 8
+    if ((tpr & 31) == 0) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) cs += __shfl_xor_sync(0xffffffffu, cs, o);
+      if ((tid & 31) == 0) atomicAdd(&s_sum[rloc], static_cast<unsigned int>(cs));
+    } else if ((tpr & (tpr - 1)) == 0) {
+      for (int o = tpr >> 1; o > 0; o >>= 1) cs += __shfl_xor_sync(0xffffffffu, cs, o);
+      if (j == 0) atomicAdd(&s_sum[rloc], static_cast<unsigned int>(cs));
+    } else {
+      atomicAdd(&s_sum[rloc], static_cast<unsigned int>(cs));
+    }
+    __syncthreads();
+    if (active && j == 0) xsum[m] = static_cast<int32_t>(s_sum[rloc]);
+  }
+}
+
+template <typename T, int kLogB, bool kStep>
+cudaError_t launch_t(const RotQuantArgs& a) {
+  constexpr int kEpt = kLogB >= 12 ? 128 : 64;
+  const int tpr = a.K / kEpt;
+  int tpb = tpr >= 128 ? tpr : (128 / tpr) * tpr;
+  if (tpb / tpr > 32) tpb = 32 * tpr;  // the per-row reduction slots hold 32 rows
+  const int rows = tpb / tpr;
+  const int grid = (a.M + rows - 1) / rows;
+  if (grid == 0) return cudaSuccess;
+  const size_t smem = (kLogB > ((kEpt == 128) ? 7 : 6)) ? static_cast<size_t>(tpb) * kEpt * sizeof(float) : 0;
+  auto kern = rotate_quant_kernel<T, kLogB, kEpt, kStep>;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  kern<<<grid, tpb, smem, a.stream>>>(reinterpret_cast<const T*>(a.x), a.M, a.K, a.inv_sqrt_b, a.step_scale, a.xq,
+                                      a.xscale, a.xsum, a.mode == 2 ? a.absmax : nullptr);
+  return cudaGetLastError();
+}
+
+template <typename T, bool kStep>
+cudaError_t launch_mode(const RotQuantArgs& a) {
+  switch (a.log_b) {
+    case 0: return launch_t<T, 0, kStep>(a);
+    case 1: return launch_t<T, 1, kStep>(a);
+    case 2: return launch_t<T, 2, kStep>(a);
+    case 3: return launch_t<T, 3, kStep>(a);
+    case 4: return launch_t<T, 4, kStep>(a);
+    case 5: return launch_t<T, 5, kStep>(a);
+    case 6: return launch_t<T, 6, kStep>(a);
+    case 7: return launch_t<T, 7, kStep>(a);
+    case 8: return launch_t<T, 8, kStep>(a);
+    case 9: return launch_t<T, 9, kStep>(a);
+    case 10: return launch_t<T, 10, kStep>(a);
+    case 11: return launch_t<T, 11, kStep>(a);
+    case 12: return launch_t<T, 12, kStep>(a);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <typename T>
+cudaError_t launch_dtype(const RotQuantArgs& a) {
+  return a.mode == 1 ? launch_mode<T, true>(a) : launch_mode<T, false>(a);
+}
+
+}  // namespace rq
+}  // namespace qvla
