@@ -191,13 +191,7 @@ def run_ours(args):
         s = {
             "gu": gu, "dn": dn,
             "x": mlp.x.to(dev),
-            "xq": torch.empty(M, K_IN // 2, dtype=torch.uint8, device=dev),
-            "xs": torch.empty(M, dtype=torch.float32, device=dev),
-            "xsum": torch.empty(M, dtype=torch.int32, device=dev),
             "h": torch.empty(M, HIDDEN, dtype=torch.bfloat16, device=dev),
-            "hq": torch.empty(M, HIDDEN // 2, dtype=torch.uint8, device=dev),
-            "hs": torch.empty(M, dtype=torch.float32, device=dev),
-            "hsum": torch.empty(M, dtype=torch.int32, device=dev),
             "y": torch.empty(M, K_IN, dtype=torch.bfloat16, device=dev),
         }
         s["ws_gu"] = torch.empty(Q.qvla_linear_workspace_bytes(gu, M), dtype=torch.uint8, device=dev)
@@ -205,20 +199,21 @@ def run_ours(args):
         sets.append(s)
 
     def step(s, ev=None):
-        # four launches: rotate+quantise x, gated gate/up GEMM, rotate+quantise h, down GEMM;
-        # ev[i] is recorded on the launching stream before launch i (ev[4] after the last)
+        # four launches, the two halves of qvla_w4a4_linear for each layer: rotate+quantise x,
+        # gated gate/up GEMM, rotate+quantise h, down GEMM; ev[i] is recorded on the launching
+        # stream before launch i (ev[4] after the last)
         if ev is not None:
             ev[0].record(stream)
-        Q.qvla_rotate_quantize(s["gu"], s["x"], M, -1, s["xq"], s["xs"], s["xsum"], stream)
+        Q.qvla_linear_quantize(s["gu"], s["x"], M, -1, s["ws_gu"], s["ws_gu"].numel(), stream)
         if ev is not None:
             ev[1].record(stream)
-        Q.qvla_gemm_w4a4(s["gu"], s["xq"], s["xs"], s["xsum"], M, s["h"], None, stream)
+        Q.qvla_linear_gemm(s["gu"], s["ws_gu"], s["ws_gu"].numel(), M, s["h"], stream)
         if ev is not None:
             ev[2].record(stream)
-        Q.qvla_rotate_quantize(s["dn"], s["h"], M, -1, s["hq"], s["hs"], s["hsum"], stream)
+        Q.qvla_linear_quantize(s["dn"], s["h"], M, -1, s["ws_dn"], s["ws_dn"].numel(), stream)
         if ev is not None:
             ev[3].record(stream)
-        Q.qvla_gemm_w4a4(s["dn"], s["hq"], s["hs"], s["hsum"], M, s["y"], None, stream)
+        Q.qvla_linear_gemm(s["dn"], s["ws_dn"], s["ws_dn"].numel(), M, s["y"], stream)
         if ev is not None:
             ev[4].record(stream)
 

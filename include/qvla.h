@@ -166,7 +166,9 @@ qvla_status qvla_rotated_absmax(const void* x, qvla_dtype xdt, int M, int K, int
 qvla_status qvla_gemm_w4a4(const qvla_layer* layer, const uint8_t* xq, const float* xscale,
                            const int32_t* xsum, int M, void* y, int32_t* acc, void* stream);
 
-/* Bytes of device workspace qvla_w4a4_linear needs for M rows (a multiple of 256). */
+/* Bytes of device workspace qvla_w4a4_linear needs for M rows (a multiple of 256): the codes
+ * travel between its two kernels as one tensor-core operand byte each (M x K bytes), plus the
+ * scales and code sums. */
 size_t qvla_linear_workspace_bytes(const qvla_layer* layer, int M);
 
 /* The whole online linear (Sec. 4): rotate + quantise x (as qvla_rotate_quantize, step as
@@ -176,6 +178,17 @@ size_t qvla_linear_workspace_bytes(const qvla_layer* layer, int M);
  * kernels on `stream` (calls that overlap on the GPU must not share it). */
 qvla_status qvla_w4a4_linear(const qvla_layer* layer, const void* x, int M, int step, void* y,
                              void* workspace, size_t workspace_bytes, void* stream);
+
+/* The two halves of qvla_w4a4_linear, for callers that schedule them separately (for example to
+ * time them, or to overlap one layer's GEMM with the next layer's rotation on another stream).
+ * qvla_linear_quantize rotates and quantises x into `workspace` (as qvla_rotate_quantize, step
+ * as there); qvla_linear_gemm then runs the integer GEMM and epilogue on it (as qvla_gemm_w4a4).
+ * The workspace contents in between are internal to the library: the codes as tensor-core
+ * operand bytes, the scales and the code sums.  Same workspace rules as qvla_w4a4_linear. */
+qvla_status qvla_linear_quantize(const qvla_layer* layer, const void* x, int M, int step, void* workspace,
+                                 size_t workspace_bytes, void* stream);
+qvla_status qvla_linear_gemm(const qvla_layer* layer, const void* workspace, size_t workspace_bytes, int M, void* y,
+                             void* stream);
 
 /* Allocation-free variant of qvla_w4a4_linear.  The paper has no counterpart: this entry
  * point exists for callers that must not allocate device memory once they are running --
@@ -190,7 +203,7 @@ qvla_status qvla_w4a4_linear(const qvla_layer* layer, const void* x, int M, int 
  * makes no cudaMalloc/cudaFree and calls no allocating library routine.  Its first call on each
  * device looks up the array's device address with that device current; make that first call
  * before any stream capture.  The scratch must hold qvla_linear_workspace_bytes(layer, M)
- * bytes (the codes [M][K/2], scales and code sums); larger requests fail with
+ * bytes (the codes [M][K] as operand bytes, scales and code sums); larger requests fail with
  * QVLA_ERR_UNSUPPORTED and enqueue nothing.  Every call shares the one array and leaves the
  * last call's contents in it; each call overwrites all it reads, so nothing needs clearing
  * in between.  Two calls whose kernels overlap on the GPU (different streams or threads, on

@@ -21,8 +21,8 @@ struct qvla_layer {
   int device = 0;
   uint8_t* wq = nullptr;      // device [N][K/2]
   float* wscale = nullptr;    // device [N]
-  int32_t* wsum = nullptr;    // device [N]
-  float* bias = nullptr;      // device [N] or null
+  float* wcorr = nullptr;     // device [N]: 8 * (sum of the codes of row n), the GEMM's offset correction
+  float* bias = nullptr;      // device [N] (zeros when the layer was given none)
   float* table = nullptr;     // device [table_cap]
   int T = 0, table_cap = 0;
 };
@@ -92,7 +92,7 @@ qvla_status check_rows(int M) {
 }
 
 qvla_status launch_rq(const void* x, int xdt, int M, int K, int had_block, int mode, const float* step_scale,
-                      uint8_t* xq, float* xscale, int32_t* xsum, float* absmax, void* stream) {
+                      uint8_t* xq, float* xscale, int32_t* xsum, float* absmax, void* stream, int out_bytes = 0) {
   qvla::RotQuantArgs a;
   a.x = x;
   a.xdt = xdt;
@@ -106,6 +106,7 @@ qvla_status launch_rq(const void* x, int xdt, int M, int K, int had_block, int m
   a.xscale = xscale;
   a.xsum = xsum;
   a.absmax = absmax;
+  a.out_bytes = out_bytes;
   a.stream = static_cast<cudaStream_t>(stream);
   QVLA_CUDA(qvla::launch_rotate_quant(a), "rotate_quantize launch");
   return QVLA_OK;
@@ -159,6 +160,12 @@ static qvla_status upload_layer(int N, int K, int had_block, qvla_dtype xdt, qvl
     if (!(wscale[n] >= 0.0f) || std::isinf(wscale[n])) return fail(QVLA_ERR_INVALID_ARG, "wscale[%d] is not a finite non-negative float", n);
   std::vector<int32_t> wsum(N);
   qvla::code_sums_host(wq, N, K, wsum.data());
+  std::vector<float> wcorr(N), zero_bias;
+  for (int n = 0; n < N; ++n) wcorr[n] = 8.0f * static_cast<float>(wsum[n]);  // exact: |8 wsum| <= 2^20
+  if (!bias) {
+    zero_bias.assign(N, 0.0f);
+    bias = zero_bias.data();
+  }
   auto* L = new (std::nothrow) qvla_layer();
   if (!L) return fail(QVLA_ERR_OOM, "host allocation failed");
   L->gated = gated;
@@ -172,12 +179,12 @@ static qvla_status upload_layer(int N, int K, int had_block, qvla_dtype xdt, qvl
   const size_t wbytes = static_cast<size_t>(N) * (K / 2);
   cudaError_t e = cudaMalloc(&L->wq, wbytes);
   if (e == cudaSuccess) e = cudaMalloc(&L->wscale, N * sizeof(float));
-  if (e == cudaSuccess) e = cudaMalloc(&L->wsum, N * sizeof(int32_t));
-  if (e == cudaSuccess && bias) e = cudaMalloc(&L->bias, N * sizeof(float));
+  if (e == cudaSuccess) e = cudaMalloc(&L->wcorr, N * sizeof(float));
+  if (e == cudaSuccess) e = cudaMalloc(&L->bias, N * sizeof(float));
   if (e == cudaSuccess) e = cudaMemcpy(L->wq, wq, wbytes, cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(L->wscale, wscale, N * sizeof(float), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess) e = cudaMemcpy(L->wsum, wsum.data(), N * sizeof(int32_t), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess && bias) e = cudaMemcpy(L->bias, bias, N * sizeof(float), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(L->wcorr, wcorr.data(), N * sizeof(float), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(L->bias, bias, N * sizeof(float), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     qvla_layer_destroy(L);
     return cuda_fail(e, "layer upload");
@@ -249,7 +256,7 @@ qvla_status qvla_layer_destroy(qvla_layer* L) {
   cudaDeviceSynchronize();
   cudaFree(L->wq);
   cudaFree(L->wscale);
-  cudaFree(L->wsum);
+  cudaFree(L->wcorr);
   cudaFree(L->bias);
   cudaFree(L->table);
   delete L;
@@ -321,21 +328,19 @@ qvla_status qvla_rotated_absmax(const void* x, qvla_dtype xdt, int M, int K, int
   return launch_rq(x, xdt, M, K, had_block, 2, nullptr, nullptr, nullptr, nullptr, absmax, stream);
 }
 
-qvla_status qvla_gemm_w4a4(const qvla_layer* L, const uint8_t* xq, const float* xscale, const int32_t* xsum, int M, void* y,
-                           int32_t* acc, void* stream) {
-  g_last_error.clear();
-  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
-  if (qvla_status s = check_rows(M)) return s;
-  if (M == 0) return QVLA_OK;
-  if (!xq || !xscale || !xsum || !y) return fail(QVLA_ERR_INVALID_ARG, "xq, xscale, xsum and y must not be NULL");
-  if (!aligned16(xq) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "xq and y must be 16-byte aligned");
+}  // extern "C"
+
+namespace {
+qvla_status launch_gemm(const qvla_layer* L, const uint8_t* xq, int x_bytes, const float* xscale, const int32_t* xsum,
+                        int M, void* y, int32_t* acc, void* stream) {
   qvla::GemmArgs a;
   a.xq = xq;
+  a.x_bytes = x_bytes;
   a.xscale = xscale;
   a.xsum = xsum;
   a.wq = L->wq;
   a.wscale = L->wscale;
-  a.wsum = L->wsum;
+  a.wcorr = L->wcorr;
   a.bias = L->bias;
   a.y = y;
   a.ydt = L->ydt;
@@ -349,10 +354,74 @@ qvla_status qvla_gemm_w4a4(const qvla_layer* L, const uint8_t* xq, const float* 
   QVLA_CUDA(qvla::launch_gemm_w4a4(a), "gemm launch");
   return QVLA_OK;
 }
+}  // namespace
+
+extern "C" {
+
+qvla_status qvla_gemm_w4a4(const qvla_layer* L, const uint8_t* xq, const float* xscale, const int32_t* xsum, int M, void* y,
+                           int32_t* acc, void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_rows(M)) return s;
+  if (M == 0) return QVLA_OK;
+  if (!xq || !xscale || !xsum || !y) return fail(QVLA_ERR_INVALID_ARG, "xq, xscale, xsum and y must not be NULL");
+  if (!aligned16(xq) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "xq and y must be 16-byte aligned");
+  return launch_gemm(L, xq, 0, xscale, xsum, M, y, acc, stream);
+}
 
 size_t qvla_linear_workspace_bytes(const qvla_layer* L, int M) {
   if (!L || M <= 0) return 0;
-  return round256(static_cast<size_t>(M) * (L->K / 2)) + round256(static_cast<size_t>(M) * 4) * 2;
+  // the codes travel between the two kernels as one operand byte each
+  return round256(static_cast<size_t>(M) * L->K) + round256(static_cast<size_t>(M) * 4) * 2;
+}
+
+namespace {
+struct LinearWorkspace {
+  uint8_t* xb;       // [M][K] operand bytes
+  float* xscale;     // [M]
+  int32_t* xsum;     // [M]
+};
+
+qvla_status carve_workspace(const qvla_layer* L, int M, void* workspace, size_t workspace_bytes, LinearWorkspace* w) {
+  if (!workspace) return fail(QVLA_ERR_INVALID_ARG, "workspace must not be NULL");
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u) return fail(QVLA_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  const size_t need = qvla_linear_workspace_bytes(L, M);
+  if (workspace_bytes < need)
+    return fail(QVLA_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed", workspace_bytes, need);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  w->xb = ws;
+  w->xscale = reinterpret_cast<float*>(ws + round256(static_cast<size_t>(M) * L->K));
+  w->xsum = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(w->xscale) + round256(static_cast<size_t>(M) * 4));
+  return QVLA_OK;
+}
+}  // namespace
+
+qvla_status qvla_linear_quantize(const qvla_layer* L, const void* x, int M, int step, void* workspace,
+                                 size_t workspace_bytes, void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_rows(M)) return s;
+  const float* ss = nullptr;
+  if (qvla_status s = resolve_step(L, step, &ss)) return s;
+  if (M == 0) return QVLA_OK;
+  if (!x) return fail(QVLA_ERR_INVALID_ARG, "x must not be NULL");
+  if (!aligned16(x)) return fail(QVLA_ERR_INVALID_ARG, "x must be 16-byte aligned");
+  LinearWorkspace w;
+  if (qvla_status s = carve_workspace(L, M, workspace, workspace_bytes, &w)) return s;
+  return launch_rq(x, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr, stream, 1);
+}
+
+qvla_status qvla_linear_gemm(const qvla_layer* L, const void* workspace, size_t workspace_bytes, int M, void* y,
+                             void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_rows(M)) return s;
+  if (M == 0) return QVLA_OK;
+  if (!y) return fail(QVLA_ERR_INVALID_ARG, "y must not be NULL");
+  if (!aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "y must be 16-byte aligned");
+  LinearWorkspace w;
+  if (qvla_status s = carve_workspace(L, M, const_cast<void*>(workspace), workspace_bytes, &w)) return s;
+  return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream);
 }
 
 qvla_status qvla_w4a4_linear(const qvla_layer* L, const void* x, int M, int step, void* y, void* workspace,
@@ -363,19 +432,13 @@ qvla_status qvla_w4a4_linear(const qvla_layer* L, const void* x, int M, int step
   const float* ss = nullptr;
   if (qvla_status s = resolve_step(L, step, &ss)) return s;
   if (M == 0) return QVLA_OK;
-  if (!x || !y || !workspace) return fail(QVLA_ERR_INVALID_ARG, "x, y and workspace must not be NULL");
+  if (!x || !y) return fail(QVLA_ERR_INVALID_ARG, "x and y must not be NULL");
   if (!aligned16(x) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "x and y must be 16-byte aligned");
-  if (reinterpret_cast<uintptr_t>(workspace) & 255u) return fail(QVLA_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
-  const size_t need = qvla_linear_workspace_bytes(L, M);
-  if (workspace_bytes < need)
-    return fail(QVLA_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed", workspace_bytes, need);
-  uint8_t* ws = static_cast<uint8_t*>(workspace);
-  uint8_t* xq = ws;
-  float* xscale = reinterpret_cast<float*>(ws + round256(static_cast<size_t>(M) * (L->K / 2)));
-  int32_t* xsum = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(xscale) + round256(static_cast<size_t>(M) * 4));
-  if (qvla_status s = launch_rq(x, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, xq, xscale, xsum, nullptr, stream))
+  LinearWorkspace w;
+  if (qvla_status s = carve_workspace(L, M, workspace, workspace_bytes, &w)) return s;
+  if (qvla_status s = launch_rq(x, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr, stream, 1))
     return s;
-  return qvla_gemm_w4a4(L, xq, xscale, xsum, M, y, nullptr, stream);
+  return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream);
 }
 
 }  // extern "C"

@@ -12,20 +12,24 @@
 // One persistent CTA per SM.  Warp roles:
 //   warps 0-3   epilogue: TMEM -> registers -> dequantise -> global (one accumulator row per thread)
 //   warp  4     TMEM allocation; lane 0 issues the MMAs and the commits
-//   warps 5-12  two producer groups of four warps, taking alternate k-blocks: they load packed
-//               nibbles from global memory, expand them to E4M3 bytes and store them in the
-//               128-byte-swizzled K-major layout the MMA descriptors expect.
-// Shared memory holds kStages k-blocks of 128 codes; TMEM holds two accumulators so the
-// epilogue of one tile overlaps the main loop of the next.
+//   warp  5     lane 0 issues TMA tensor loads of packed int4 tiles into a staging ring
+//   warps 6-13  converters: staged nibbles -> E4M3 bytes in the 128-byte-swizzled K-major
+//               layout the MMA descriptors expect
+// Shared memory holds kStages staged (packed) and kStages expanded k-blocks of 128 codes; TMEM
+// holds two accumulators so the epilogue of one tile overlaps the main loop of the next.  The epilogue stages each tile's
+// per-column parameters (weight scale, weight-code correction, bias) in shared memory.
 //
 // Two orientations: for M > 128 the MMA's M side is the activations (tile 128 tokens x 256
 // weight rows); for M <= 128 ("swap") it is the weights (128 weight rows x Mpad tokens),
 // so that a small batch does not waste the 128-row MMA.
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 
 #include <cstdint>
+#include <mutex>
 
 #include "kernels.h"
 #include "ptx.cuh"
@@ -36,22 +40,30 @@ namespace {
 constexpr int kBM = 128;        // MMA M (rows of the MMA A operand)
 constexpr int kBK = 128;        // codes per k-block (one 128-byte swizzle row of E4M3)
 constexpr int kEpiWarps = 4;
+constexpr int kEpiThreads = kEpiWarps * 32;
 constexpr int kMmaWarp = 4;
-constexpr int kProdWarpsPerGroup = 4;
-constexpr int kProdGroups = 2;
-constexpr int kProdThreadsPerGroup = kProdWarpsPerGroup * 32;
-constexpr int kThreads = (kEpiWarps + 1 + kProdGroups * kProdWarpsPerGroup) * 32;
+constexpr int kTmaWarp = 5;
+constexpr int kConvWarps = 8;
+constexpr int kConvThreads = kConvWarps * 32;
+constexpr int kThreads = (kEpiWarps + 2 + kConvWarps) * 32;
+constexpr uint32_t kEpiBarrier = 1;  // named barrier of the epilogue warps
 
-template <int kBN>
+// kStageA / kStageB: whether operand A / B of the MMA arrives packed (staged, then expanded by
+// the converters); otherwise it arrives as operand bytes straight from a swizzled TMA load.
+template <int kBN, bool kStageA = true, bool kStageB = true>
 struct Cfg {
   static constexpr int kTileA = kBM * kBK;    // bytes of E4M3
   static constexpr int kTileB = kBN * kBK;
-  static constexpr int kStage = kTileA + kTileB;
-  static constexpr int kStagesRaw = (200 * 1024) / kStage;
+  static constexpr int kStage = kTileA + kTileB;             // expanded k-block
+  static constexpr int kRawA = kStageA ? kBM * kBK / 2 : 0;  // packed k-block (64-byte rows)
+  static constexpr int kRawB = kStageB ? kBN * kBK / 2 : 0;
+  static constexpr int kRaw = kRawA + kRawB;
+  static constexpr int kStagesRaw = (216 * 1024) / (kStage + kRaw);
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
-  static constexpr int kSmem = kStages * kStage + 1024;  // + alignment slack
+  static constexpr int kSmem = kStages * (kStage + kRaw) + 1024;  // + alignment slack
   static constexpr uint32_t kTmemCols = (2 * kBN) <= 32 ? 32 : (2 * kBN) <= 64 ? 64 : (2 * kBN) <= 128 ? 128 : (2 * kBN) <= 256 ? 256 : 512;
   static_assert(kStages >= 2, "stages");
+  static_assert(kRaw % 1024 == 0 && kStage % 1024 == 0, "1024-byte aligned stages");
 };
 
 struct Params {
@@ -60,35 +72,31 @@ struct Params {
   int rows_a, rows_b, K;
   const float* xscale;
   const int32_t* xsum;
-  const float* wscale;
-  const int32_t* wsum;
-  const float* bias;
+  const float* wscale;  // [N]
+  const float* wcorr;   // [N] 8 * sum_k qw[n,k]
+  const float* bias;    // [N] (zeros when the layer has none)
   void* y;
   int32_t* acc;
   int M, N;      // N = weight rows of the layer (2H for a gated layer)
   int ldy;       // row length of y (N, or H for a gated layer)
 };
 
-__device__ __forceinline__ uint4 ldg_nc(const uint8_t* p) {
-  uint4 r;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-               : "l"(p));
-  return r;
+__device__ __forceinline__ void epi_sync() {
+  asm volatile("bar.sync %0, %1;" ::"n"(kEpiBarrier), "n"(kEpiThreads) : "memory");
 }
 
-// Expand one 16-byte chunk (32 codes) into 32 E4M3 bytes and store them as the two 16-byte
-// columns 2q and 2q+1 of row r of a 128-byte-swizzled tile.
-__device__ __forceinline__ void store_chunk(uint8_t* tile, int r, int q, uint4 v) {
+// Expand one 16-byte chunk (32 codes) into 32 E4M3 bytes at row + the two swizzled 16-byte
+// columns o0 and o1 of a 128-byte-swizzled tile row.  The byte order inside each group of 8
+// codes becomes (0,2,4,6,1,3,5,7); both operands get the same order, so the dot product over
+// k is unchanged.
+__device__ __forceinline__ void store_chunk(uint8_t* row, int o0, int o1, uint4 v) {
   uint32_t o[8];
   int4x8_to_e4m3_offset(v.x, o[0], o[1]);
   int4x8_to_e4m3_offset(v.y, o[2], o[3]);
   int4x8_to_e4m3_offset(v.z, o[4], o[5]);
   int4x8_to_e4m3_offset(v.w, o[6], o[7]);
-  uint8_t* row = tile + r * 128;
-  const int sw = r & 7;
-  *reinterpret_cast<uint4*>(row + (((2 * q) ^ sw) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
-  *reinterpret_cast<uint4*>(row + (((2 * q + 1) ^ sw) << 4)) = make_uint4(o[4], o[5], o[6], o[7]);
+  *reinterpret_cast<uint4*>(row + o0) = make_uint4(o[0], o[1], o[2], o[3]);
+  *reinterpret_cast<uint4*>(row + o1) = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
 // GELU, tanh form, written as g * sigmoid(2u) = g / (1 + exp(-2u)), u = sqrt(2/pi) (g + 0.044715 g^3):
@@ -98,40 +106,77 @@ __device__ __forceinline__ float gelu_tanh(float g) {
   return __fdividef(g, 1.0f + __expf(-2.0f * u));
 }
 
+// Two floats rounded to the output dtype (one pair conversion), as raw bits.
+template <typename OutT>
+__device__ __forceinline__ uint32_t pack2(float a, float b);
+template <>
+__device__ __forceinline__ uint32_t pack2<__half>(float a, float b) {
+  __half2 h = __floats2half2_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+template <>
+__device__ __forceinline__ uint32_t pack2<__nv_bfloat16>(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+// The two values of a pair, back to float.
+template <typename OutT>
+__device__ __forceinline__ float2 unpack2(uint32_t v);
+template <>
+__device__ __forceinline__ float2 unpack2<__half>(uint32_t v) {
+  return __half22float2(*reinterpret_cast<__half2*>(&v));
+}
+template <>
+__device__ __forceinline__ float2 unpack2<__nv_bfloat16>(uint32_t v) {
+  return make_float2(__uint_as_float(v << 16), __uint_as_float(v & 0xFFFF0000u));
+}
 template <typename OutT>
 __device__ __forceinline__ OutT to_out(float v);
 template <>
 __device__ __forceinline__ __half to_out<__half>(float v) { return __float2half_rn(v); }
 template <>
 __device__ __forceinline__ __nv_bfloat16 to_out<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
-__device__ __forceinline__ float from_out(__half v) { return __half2float(v); }
-__device__ __forceinline__ float from_out(__nv_bfloat16 v) { return __bfloat162float(v); }
 
-// 32 outputs of one row as 4 x 16-byte stores (or element stores at a ragged edge).
+// 32 outputs (16 packed pairs) of one row: 4 x 16-byte stores, or element stores at a ragged edge.
 template <typename OutT>
-__device__ __forceinline__ void store_row32(OutT* dst, const OutT (&out)[32], int nvalid) {
+__device__ __forceinline__ void store_row32(OutT* dst, const uint32_t (&pk)[16], int nvalid) {
   if (nvalid == 32) {
-    const uint4* src = reinterpret_cast<const uint4*>(out);
     uint4* d = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-    for (int i = 0; i < 4; ++i) d[i] = src[i];
+    for (int i = 0; i < 4; ++i) d[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
   } else {
-    for (int i = 0; i < nvalid; ++i) dst[i] = out[i];
+    uint16_t* d = reinterpret_cast<uint16_t*>(dst);
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (i < nvalid) d[i] = static_cast<uint16_t>(pk[i >> 1] >> (16 * (i & 1)));
   }
 }
 
-template <int kBN, bool kSwap, bool kGated, typename OutT>
-__global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(Params p) {
-  using C = Cfg<kBN>;
+// kXBytes: the activations arrive as operand bytes ([rows][K], written by the rotate-quantise
+// kernel) and are TMA-loaded with the 128-byte swizzle straight into the MMA operand tile; only
+// the weights are staged and expanded.  Otherwise both operands are packed int4.
+template <int kBN, bool kSwap, bool kGated, bool kXBytes, typename OutT>
+__global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_constant__ CUtensorMap tmap_a,
+                                                                 const __grid_constant__ CUtensorMap tmap_b, Params p) {
+  constexpr bool kStageA = !(kXBytes && !kSwap);  // operand A is the activations unless swapped
+  constexpr bool kStageB = !(kXBytes && kSwap);
+  using C = Cfg<kBN, kStageA, kStageB>;
   extern __shared__ uint8_t dyn_smem[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~uintptr_t(1023));
 
-  __shared__ __align__(8) uint64_t bar_full[C::kStages];
-  __shared__ __align__(8) uint64_t bar_empty[C::kStages];
+  __shared__ __align__(8) uint64_t bar_raw_full[C::kStages];   // TMA bytes landed
+  __shared__ __align__(8) uint64_t bar_raw_empty[C::kStages];  // converters done with the staged k-block
+  __shared__ __align__(8) uint64_t bar_full[C::kStages];       // expanded k-block ready for the MMA
+  __shared__ __align__(8) uint64_t bar_empty[C::kStages];      // MMAs done reading it
   __shared__ __align__(8) uint64_t bar_tfull[2];
   __shared__ __align__(8) uint64_t bar_tempty[2];
   __shared__ __align__(8) uint64_t bar_done;
   __shared__ uint32_t s_tmem_base;
+  __shared__ int s_epi_abort;  // set by an epilogue thread whose wait timed out
+  // per-column parameters of the current tile (non-swap): weight scale, code correction, bias
+  __shared__ __align__(16) float s_ws[kSwap ? 1 : kBN];
+  __shared__ __align__(16) float s_wc[kSwap ? 1 : kBN];
+  __shared__ __align__(16) float s_bs[kSwap ? 1 : kBN];
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -140,19 +185,22 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(Params p) {
   const int tiles_b = (p.rows_b + kBN - 1) / kBN;
   const int ntiles = tiles_a * tiles_b;
   const int nkb = p.K / kBK;
-  const int kbytes = p.K / 2;
+  uint8_t* const raw = smem + C::kStages * C::kStage;  // staging ring after the expanded stages
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
-      mbar_init(smem_u32(&bar_full[s]), kProdThreadsPerGroup);
+      mbar_init(smem_u32(&bar_raw_full[s]), 1);
+      mbar_init(smem_u32(&bar_raw_empty[s]), kConvThreads);
+      mbar_init(smem_u32(&bar_full[s]), kConvThreads + (kXBytes ? 1 : 0));  // + the TMA thread's byte count
       mbar_init(smem_u32(&bar_empty[s]), 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&bar_tfull[i]), 1);
-      mbar_init(smem_u32(&bar_tempty[i]), kEpiWarps * 32);
+      mbar_init(smem_u32(&bar_tempty[i]), kEpiThreads);
     }
     mbar_init(smem_u32(&bar_done), 1);
     mbar_init_fence();
+    s_epi_abort = 0;
   }
   if (warp == kMmaWarp) tmem_alloc<C::kTmemCols>(smem_u32(&s_tmem_base));
   tc_fence_before();
@@ -160,51 +208,84 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(Params p) {
   tc_fence_after();
   const uint32_t tmem_base = s_tmem_base;
 
-  if (warp >= kMmaWarp + 1) {
-    // ------------------------------------------------------------------ producers
-    const int g = (warp - (kMmaWarp + 1)) / kProdWarpsPerGroup;
-    const int pt = threadIdx.x - (kMmaWarp + 1) * 32 - g * kProdThreadsPerGroup;
-    constexpr int kChunksA = kBM * 4;   // 16-byte packed chunks per A tile
-    constexpr int kChunksB = kBN * 4;
-    constexpr int kPerThreadA = kChunksA / kProdThreadsPerGroup;
-    constexpr int kPerThreadB = (kChunksB + kProdThreadsPerGroup - 1) / kProdThreadsPerGroup;
+  if (warp == kTmaWarp) {
+    // ------------------------------------------------------------------ TMA loads of packed tiles
+    if (lane == 0) {
+      tma_prefetch_desc(&tmap_a);
+      tma_prefetch_desc(&tmap_b);
+      int it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+        const int ta = tile % tiles_a, tb = tile / tiles_a;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = it % C::kStages;
+          const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
+          if (!mbar_wait(smem_u32(&bar_raw_empty[s]), ph ^ 1u)) { ok = false; break; }
+          const uint32_t bar = smem_u32(&bar_raw_full[s]);
+          mbar_arrive_expect_tx(bar, C::kRaw);
+          const uint32_t dst = smem_u32(raw + s * C::kRaw);
+          if constexpr (kStageA) tma_load_2d(dst, &tmap_a, kb * (kBK / 2), ta * kBM, bar);
+          if constexpr (kStageB) tma_load_2d(dst + C::kRawA, &tmap_b, kb * (kBK / 2), tb * kBN, bar);
+          if constexpr (kXBytes) {
+            // the activation operand goes straight into the expanded stage once the MMAs are done with it
+            if (!mbar_wait(smem_u32(&bar_empty[s]), ph ^ 1u)) { ok = false; break; }
+            const uint32_t fb = smem_u32(&bar_full[s]);
+            const uint32_t e = smem_u32(smem + s * C::kStage);
+            if constexpr (!kSwap) {
+              mbar_arrive_expect_tx(fb, C::kTileA);
+              tma_load_2d(e, &tmap_a, kb * kBK, ta * kBM, fb);
+            } else {
+              mbar_arrive_expect_tx(fb, C::kTileB);
+              tma_load_2d(e + C::kTileA, &tmap_b, kb * kBK, tb * kBN, fb);
+            }
+          }
+        }
+      }
+      // before leaving, let every load issued above land (a no-op unless a wait timed out)
+      for (int k = 0; k < C::kStages && k < it; ++k) {
+        const int j = it - 1 - k;
+        mbar_wait(smem_u32(&bar_raw_full[j % C::kStages]), static_cast<uint32_t>(j / C::kStages) & 1u);
+      }
+    }
+    __syncwarp();
+  } else if (warp > kTmaWarp) {
+    // ------------------------------------------------------------------ converters
+    const int ct = threadIdx.x - (kTmaWarp + 1) * 32;  // 0 .. kConvThreads-1
+    constexpr int kChunksA = kStageA ? kBM * 4 : 0;     // 16-byte packed chunks per k-block
+    constexpr int kChunks = kChunksA + (kStageB ? kBN * 4 : 0);
+    constexpr int kPer = (kChunks + kConvThreads - 1) / kConvThreads;
+    // destination of each of this thread's chunks: tile byte offset of the row and the two
+    // swizzled 16-byte columns; the staged chunk c sits at byte 16 c of the staging k-block
+    int d_row[kPer], d_o0[kPer], d_o1[kPer];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+      const int c = ct + i * kConvThreads;
+      const int cc = c < kChunksA ? c : c - kChunksA;
+      const int r = cc >> 2, q = cc & 3;
+      d_row[i] = (c < kChunksA ? 0 : C::kTileA) + r * 128;
+      d_o0[i] = ((2 * q) ^ (r & 7)) << 4;
+      d_o1[i] = ((2 * q + 1) ^ (r & 7)) << 4;
+    }
     int it = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-      const int ta = tile % tiles_a, tb = tile / tiles_a;
       for (int kb = 0; kb < nkb; ++kb, ++it) {
-        if ((it & 1) != g) continue;
         const int s = it % C::kStages;
         const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
-        uint4 va[kPerThreadA], vb[kPerThreadB];
-#pragma unroll
-        for (int i = 0; i < kPerThreadA; ++i) {
-          const int c = pt + i * kProdThreadsPerGroup;
-          const int row = ta * kBM + (c >> 2);
-          va[i] = row < p.rows_a ? ldg_nc(p.a + static_cast<size_t>(row) * kbytes + kb * 64 + (c & 3) * 16)
-                                 : make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);
-        }
-#pragma unroll
-        for (int i = 0; i < kPerThreadB; ++i) {
-          const int c = pt + i * kProdThreadsPerGroup;
-          const int row = tb * kBN + (c >> 2);
-          vb[i] = (c < kChunksB && row < p.rows_b)
-                      ? ldg_nc(p.b + static_cast<size_t>(row) * kbytes + kb * 64 + (c & 3) * 16)
-                      : make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);
-        }
+        if (!mbar_wait(smem_u32(&bar_raw_full[s]), ph)) { ok = false; break; }
         if (!mbar_wait(smem_u32(&bar_empty[s]), ph ^ 1u)) { ok = false; break; }
-        uint8_t* sa = smem + s * C::kStage;
-        uint8_t* sb = sa + C::kTileA;
+        const uint8_t* src = raw + s * C::kRaw;
+        uint8_t* dst = smem + s * C::kStage;
+        uint4 v[kPer];
 #pragma unroll
-        for (int i = 0; i < kPerThreadA; ++i) {
-          const int c = pt + i * kProdThreadsPerGroup;
-          store_chunk(sa, c >> 2, c & 3, va[i]);
-        }
+        for (int i = 0; i < kPer; ++i)
+          if (kChunks % kConvThreads == 0 || ct + i * kConvThreads < kChunks)
+            v[i] = *reinterpret_cast<const uint4*>(src + 16 * (ct + i * kConvThreads));
+        mbar_arrive(smem_u32(&bar_raw_empty[s]));  // the staged k-block is in registers now
 #pragma unroll
-        for (int i = 0; i < kPerThreadB; ++i) {
-          const int c = pt + i * kProdThreadsPerGroup;
-          if (c < kChunksB) store_chunk(sb, c >> 2, c & 3, vb[i]);
-        }
+        for (int i = 0; i < kPer; ++i)
+          if (kChunks % kConvThreads == 0 || ct + i * kConvThreads < kChunks)
+            store_chunk(dst + d_row[i], d_o0[i], d_o1[i], v[i]);
         fence_proxy_async_smem();
         mbar_arrive(smem_u32(&bar_full[s]));
       }
@@ -252,7 +333,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(Params p) {
       const int ta = tile % tiles_a, tb = tile / tiles_a;
       const int buf = tile_iter & 1;
       const uint32_t aph = static_cast<uint32_t>(tile_iter >> 1) & 1u;
-      if (!mbar_wait(smem_u32(&bar_tfull[buf]), aph)) break;
+      // All epilogue threads pass this barrier every tile, so the abort decision below is
+      // uniform and no thread is left waiting at a named barrier.  It also tells the writers
+      // of the column parameters that the previous tile's readers are done.
+      epi_sync();
+      if (s_epi_abort) break;
+      if constexpr (!kSwap) {
+        // stage this tile's column parameters while the accumulator is still being computed
+        for (int c = et; c < kBN; c += kEpiThreads) {
+          const int n = min(tb * kBN + c, p.N - 1);
+          s_ws[c] = __ldg(p.wscale + n);
+          s_wc[c] = __ldg(p.wcorr + n);
+          s_bs[c] = __ldg(p.bias + n);
+        }
+        epi_sync();
+      }
+      if (!mbar_wait(smem_u32(&bar_tfull[buf]), aph)) {
+        s_epi_abort = 1;
+        continue;
+      }
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(warp * 32) << 16) + static_cast<uint32_t>(buf * kBN);
       const int ra = ta * kBM + et;  // this thread's MMA-A row
@@ -272,21 +371,31 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(Params p) {
           const int n0 = tb * kBN + c0;
           if (mok && n0 < p.N) {
             const int nvalid = min(32, p.N - n0);
-            alignas(16) OutT out[32];
-            int32_t ai[32];
+            float acc[32];
+            uint32_t pk[16];
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int n = min(n0 + i, p.N - 1);
-              const float corr = cm + 8.0f * static_cast<float>(__ldg(p.wsum + n));
-              const float acc = fmaf(__uint_as_float(r[i]), 262144.0f, -corr);
-              const float b = p.bias ? __ldg(p.bias + n) : 0.0f;
-              out[i] = to_out<OutT>(fmaf(acc, xs * __ldg(p.wscale + n), b));
-              ai[i] = static_cast<int32_t>(acc);
+            for (int i4 = 0; i4 < 8; ++i4) {
+              const float4 ws = *reinterpret_cast<const float4*>(s_ws + c0 + 4 * i4);
+              const float4 wc = *reinterpret_cast<const float4*>(s_wc + c0 + 4 * i4);
+              const float4 bs = *reinterpret_cast<const float4*>(s_bs + c0 + 4 * i4);
+              const float wsv[4] = {ws.x, ws.y, ws.z, ws.w}, wcv[4] = {wc.x, wc.y, wc.z, wc.w};
+              const float bsv[4] = {bs.x, bs.y, bs.z, bs.w};
+              float yv[4];
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const int i = 4 * i4 + k;
+                acc[i] = fmaf(__uint_as_float(r[i]), 262144.0f, -(cm + wcv[k]));
+                yv[k] = fmaf(acc[i], xs * wsv[k], bsv[k]);
+              }
+              pk[2 * i4] = pack2<OutT>(yv[0], yv[1]);
+              pk[2 * i4 + 1] = pack2<OutT>(yv[2], yv[3]);
             }
-            store_row32(yrow + n0, out, nvalid);
+            store_row32(yrow + n0, pk, nvalid);
             if (p.acc) {
               int32_t* arow = p.acc + static_cast<size_t>(m) * p.N + n0;
-              for (int i = 0; i < nvalid; ++i) arow[i] = ai[i];
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (i < nvalid) arow[i] = static_cast<int32_t>(acc[i]);
             }
           }
         }
@@ -304,29 +413,47 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(Params p) {
         const int H = p.N / 2;
         OutT* yrow = reinterpret_cast<OutT*>(p.y) + static_cast<size_t>(mok ? m : 0) * p.ldy;
 #pragma unroll 1
-        for (int c0 = 0; c0 < kHalf; c0 += 32) {
-          uint32_t rg[32], ru[32];
+        for (int c0 = 0; c0 < kHalf; c0 += 16) {
+          uint32_t rg[16], ru[16];
           __syncwarp();
-          tmem_ld32(taddr + c0, rg);
-          tmem_ld32(taddr + kHalf + c0, ru);
+          tmem_ld16(taddr + c0, rg);
+          tmem_ld16(taddr + kHalf + c0, ru);
           tmem_ld_wait();
           if (mok) {
-            alignas(16) OutT out[32];
+            uint32_t pk[8];
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int ng = tb * kBN + c0 + i, nu = ng + kHalf;
-              const float ag = fmaf(__uint_as_float(rg[i]), 262144.0f, -(cm + 8.0f * static_cast<float>(__ldg(p.wsum + ng))));
-              const float au = fmaf(__uint_as_float(ru[i]), 262144.0f, -(cm + 8.0f * static_cast<float>(__ldg(p.wsum + nu))));
-              const float g = from_out(to_out<OutT>(fmaf(ag, xs * __ldg(p.wscale + ng), p.bias ? __ldg(p.bias + ng) : 0.0f)));
-              const float u = from_out(to_out<OutT>(fmaf(au, xs * __ldg(p.wscale + nu), p.bias ? __ldg(p.bias + nu) : 0.0f)));
-              out[i] = to_out<OutT>(gelu_tanh(g) * u);
-              if (p.acc) {  // debug view in natural order: [gate units | up units]
-                int32_t* arow = p.acc + static_cast<size_t>(m) * p.N;
-                arow[j0 + c0 + i] = static_cast<int32_t>(ag);
-                arow[H + j0 + c0 + i] = static_cast<int32_t>(au);
+            for (int i4 = 0; i4 < 4; ++i4) {
+              const int cg = c0 + 4 * i4, cu = cg + kHalf;
+              const float4 wsg = *reinterpret_cast<const float4*>(s_ws + cg);
+              const float4 wcg = *reinterpret_cast<const float4*>(s_wc + cg);
+              const float4 bsg = *reinterpret_cast<const float4*>(s_bs + cg);
+              const float4 wsu = *reinterpret_cast<const float4*>(s_ws + cu);
+              const float4 wcu = *reinterpret_cast<const float4*>(s_wc + cu);
+              const float4 bsu = *reinterpret_cast<const float4*>(s_bs + cu);
+              const float wsgv[4] = {wsg.x, wsg.y, wsg.z, wsg.w}, wcgv[4] = {wcg.x, wcg.y, wcg.z, wcg.w};
+              const float bsgv[4] = {bsg.x, bsg.y, bsg.z, bsg.w}, wsuv[4] = {wsu.x, wsu.y, wsu.z, wsu.w};
+              const float wcuv[4] = {wcu.x, wcu.y, wcu.z, wcu.w}, bsuv[4] = {bsu.x, bsu.y, bsu.z, bsu.w};
+              float hv[4];
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const int i = 4 * i4 + k;
+                const float ag = fmaf(__uint_as_float(rg[i]), 262144.0f, -(cm + wcgv[k]));
+                const float au = fmaf(__uint_as_float(ru[i]), 262144.0f, -(cm + wcuv[k]));
+                // gate and up rounded to the output dtype (one pair conversion), then h
+                const float2 gu = unpack2<OutT>(pack2<OutT>(fmaf(ag, xs * wsgv[k], bsgv[k]), fmaf(au, xs * wsuv[k], bsuv[k])));
+                hv[k] = gelu_tanh(gu.x) * gu.y;
+                if (p.acc) {  // debug view in natural order: [gate units | up units]
+                  int32_t* arow = p.acc + static_cast<size_t>(m) * p.N;
+                  arow[j0 + c0 + i] = static_cast<int32_t>(ag);
+                  arow[H + j0 + c0 + i] = static_cast<int32_t>(au);
+                }
               }
+              pk[2 * i4] = pack2<OutT>(hv[0], hv[1]);
+              pk[2 * i4 + 1] = pack2<OutT>(hv[2], hv[3]);
             }
-            store_row32(yrow + j0 + c0, out, 32);
+            uint4* d = reinterpret_cast<uint4*>(yrow + j0 + c0);
+            d[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            d[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
           }
         }
       } else {
@@ -334,8 +461,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(Params p) {
         const int n = ra;
         const bool nok = n < p.N;
         const float ws = nok ? __ldg(p.wscale + n) : 0.0f;
-        const float cn = nok ? 8.0f * static_cast<float>(__ldg(p.wsum + n)) + k64 : 0.0f;
-        const float b = (nok && p.bias) ? __ldg(p.bias + n) : 0.0f;
+        const float cn = nok ? __ldg(p.wcorr + n) + k64 : 0.0f;
+        const float b = nok ? __ldg(p.bias + n) : 0.0f;
         constexpr int kChunk = kBN < 32 ? kBN : 32;
 #pragma unroll 1
         for (int c0 = 0; c0 < kBN; c0 += kChunk) {
@@ -374,9 +501,54 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(Params p) {
   if (warp == kMmaWarp) tmem_dealloc<C::kTmemCols>(tmem_base);
 }
 
-template <int kBN, bool kSwap, bool kGated, typename OutT>
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// A [rows][row_bytes] byte matrix read in boxes of 64 bytes (one k-block of packed codes) x
+// box_rows rows; rows past the end read as zero.
+cudaError_t make_tmap(CUtensorMap* m, const void* base, int rows, int row_bytes, int box_rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (!enc) return cudaErrorNotSupported;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(row_bytes), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(row_bytes)};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK / 2), static_cast<cuuint32_t>(box_rows)};
+  const cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+// An operand for the swizzled direct load: [rows][K] operand bytes in boxes of 128 bytes (one
+// k-block) x box_rows, written into shared memory with the 128-byte swizzle of the MMA layout.
+cudaError_t make_tmap_bytes(CUtensorMap* m, const void* base, int rows, int K, int box_rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (!enc) return cudaErrorNotSupported;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(box_rows)};
+  const cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+template <int kBN, bool kSwap, bool kGated, bool kXBytes, typename OutT>
 cudaError_t launch_cfg(const GemmArgs& a) {
-  using C = Cfg<kBN>;
+  constexpr bool kStageA = !(kXBytes && !kSwap);
+  constexpr bool kStageB = !(kXBytes && kSwap);
+  using C = Cfg<kBN, kStageA, kStageB>;
   Params p;
   if (kSwap) {
     p.a = a.wq;
@@ -393,7 +565,7 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   p.xscale = a.xscale;
   p.xsum = a.xsum;
   p.wscale = a.wscale;
-  p.wsum = a.wsum;
+  p.wcorr = a.wcorr;
   p.bias = a.bias;
   p.y = a.y;
   p.acc = a.acc;
@@ -403,29 +575,35 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   const int tiles = ((p.rows_a + kBM - 1) / kBM) * ((p.rows_b + kBN - 1) / kBN);
   const int grid = tiles < a.num_sms ? tiles : a.num_sms;
   if (grid == 0) return cudaSuccess;
-  auto kern = gemm_w4a4_kernel<kBN, kSwap, kGated, OutT>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+  CUtensorMap ta, tb;
+  cudaError_t e = kStageA ? make_tmap(&ta, p.a, p.rows_a, p.K / 2, kBM) : make_tmap_bytes(&ta, p.a, p.rows_a, p.K, kBM);
+  if (e == cudaSuccess)
+    e = kStageB ? make_tmap(&tb, p.b, p.rows_b, p.K / 2, kBN) : make_tmap_bytes(&tb, p.b, p.rows_b, p.K, kBN);
   if (e != cudaSuccess) return e;
-  kern<<<grid, kThreads, C::kSmem, a.stream>>>(p);
+  auto kern = gemm_w4a4_kernel<kBN, kSwap, kGated, kXBytes, OutT>;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+  if (e != cudaSuccess) return e;
+  kern<<<grid, kThreads, C::kSmem, a.stream>>>(ta, tb, p);
   return cudaGetLastError();
 }
 
-template <typename OutT>
+template <bool kXBytes, typename OutT>
 cudaError_t launch_out(const GemmArgs& a) {
-  if (a.gated) return launch_cfg<256, false, true, OutT>(a);  // gate/up pairs share a 256-row tile
-  if (a.M > 128) return launch_cfg<256, false, false, OutT>(a);
+  if (a.gated) return launch_cfg<256, false, true, kXBytes, OutT>(a);  // gate/up pairs share a 256-row tile
+  if (a.M > 128) return launch_cfg<256, false, false, kXBytes, OutT>(a);
   const int mpad = (a.M + 15) / 16 * 16;
-  if (mpad <= 16) return launch_cfg<16, true, false, OutT>(a);
-  if (mpad <= 32) return launch_cfg<32, true, false, OutT>(a);
-  if (mpad <= 64) return launch_cfg<64, true, false, OutT>(a);
-  return launch_cfg<128, true, false, OutT>(a);
+  if (mpad <= 16) return launch_cfg<16, true, false, kXBytes, OutT>(a);
+  if (mpad <= 32) return launch_cfg<32, true, false, kXBytes, OutT>(a);
+  if (mpad <= 64) return launch_cfg<64, true, false, kXBytes, OutT>(a);
+  return launch_cfg<128, true, false, kXBytes, OutT>(a);
 }
 
 }  // namespace
 
 cudaError_t launch_gemm_w4a4(const GemmArgs& a) {
   if (a.M == 0) return cudaSuccess;
-  return a.ydt == 0 ? launch_out<__half>(a) : launch_out<__nv_bfloat16>(a);
+  if (a.x_bytes) return a.ydt == 0 ? launch_out<true, __half>(a) : launch_out<true, __nv_bfloat16>(a);
+  return a.ydt == 0 ? launch_out<false, __half>(a) : launch_out<false, __nv_bfloat16>(a);
 }
 
 cudaError_t read_and_clear_error_word(unsigned int* out, cudaStream_t stream) {

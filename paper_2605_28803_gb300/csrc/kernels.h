@@ -17,7 +17,8 @@ struct RotQuantArgs {
   float inv_sqrt_b;        // float32(1 / sqrt(b))
   int mode;                // 0 per-token, 1 per-step (step_scale), 2 absmax only
   const float* step_scale; // device, one float (mode 1)
-  uint8_t* xq;             // device [M][K/2]
+  uint8_t* xq;             // device [M][K/2] packed codes, or [M][K] operand bytes (out_bytes)
+  int out_bytes;           // 1: one E4M3 operand byte per code (the GEMM's internal encoding)
   float* xscale;           // device [M]
   int32_t* xsum;           // device [M] or null
   float* absmax;           // device, one float (mode 2)
@@ -28,13 +29,14 @@ cudaError_t launch_rotate_quant(const RotQuantArgs& a);
 
 // ---- W4A4 GEMM + epilogue (gemm.cu) ----
 struct GemmArgs {
-  const uint8_t* xq;       // device [M][K/2] activation codes
+  const uint8_t* xq;       // device [M][K/2] activation codes, or [M][K] operand bytes (x_bytes)
+  int x_bytes;             // 1: xq holds the rotate-quantise kernel's operand bytes
   const float* xscale;     // device [M]
   const int32_t* xsum;     // device [M]
   const uint8_t* wq;       // device [N][K/2] weight codes
   const float* wscale;     // device [N]
-  const int32_t* wsum;     // device [N]
-  const float* bias;       // device [N] or null
+  const float* wcorr;      // device [N]: 8 * sum_k wq[n,k] as float
+  const float* bias;       // device [N] (zeros when the layer has no bias)
   void* y;                 // device [M][N], dtype ydt
   int ydt;                 // 0 f16, 1 bf16
   int32_t* acc;            // device [M][N] or null

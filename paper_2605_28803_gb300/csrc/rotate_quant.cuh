@@ -136,7 +136,8 @@ template <typename T, int kLogB, int kEpt, bool kStep>
 __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__ x, int M, int K, float inv_sqrt_b,
                                                              const float* __restrict__ step_scale,
                                                              uint8_t* __restrict__ xq, float* __restrict__ xscale,
-                                                             int32_t* __restrict__ xsum, float* __restrict__ absmax_out) {
+                                                             int32_t* __restrict__ xsum, float* __restrict__ absmax_out,
+                                                             int out_bytes) {
   constexpr int kP = (kEpt == 128) ? 7 : 6;  // log2(kEpt)
   static_assert((1 << kP) == kEpt, "EPT");
   constexpr int kN = kEpt / 2;                // float2 per thread
@@ -273,7 +274,7 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
   }
 
   // ---- store: run r holds register elements [r kRun, (r + 1) kRun), contiguous in the row ----
-  if (active) {
+  if (active && !out_bytes) {  // packed nibbles [M][K/2]
     uint8_t* dst = xq + static_cast<size_t>(m) * (K / 2);
 #pragma unroll
     for (int run = 0; run < kEpt / kRun; ++run) {
@@ -299,6 +300,44 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
         for (int w = 0; w < kBytes / 4; w += 4)
           *reinterpret_cast<uint4*>(p + 4 * w) =
               make_uint4(pk[(b0 >> 2) + w], pk[(b0 >> 2) + w + 1], pk[(b0 >> 2) + w + 2], pk[(b0 >> 2) + w + 3]);
+      }
+    }
+  } else if (active) {
+    // One byte per code, the GEMM's tensor-core operand encoding: code q as the E4M3 byte
+    // q + 8 (= q XOR 8).  Within each group of 8 consecutive k the bytes are stored in the order
+    // k0 k2 k4 k6 k1 k3 k5 k7 -- the order the GEMM gives the packed operand it expands -- so
+    // both operands of the dot product agree.
+    uint8_t* dst = xq + static_cast<size_t>(m) * K;
+    uint32_t lo[kEpt / 8], hi[kEpt / 8];
+#pragma unroll
+    for (int g = 0; g < kEpt / 8; ++g) {
+      lo[g] = (pk[g] ^ 0x88888888u) & 0x0F0F0F0Fu;          // even elements of the 8
+      hi[g] = ((pk[g] >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;   // odd elements
+    }
+#pragma unroll
+    for (int run = 0; run < kEpt / kRun; ++run) {
+      int e0;
+      if constexpr (kPhase2) {
+        e0 = ((j >> kR) << kLogB) | (run << kP) | ((j & ((1 << kR) - 1)) << kL);
+      } else {
+        e0 = j * kEpt;
+      }
+      uint8_t* gb = dst + (e0 & ~7);  // the 8-byte group this run starts in
+      const int o = e0 & 7;
+      if constexpr (kRun >= 8) {
+#pragma unroll
+        for (int t = 0; t < kRun / 8; ++t) {
+          const int w = run * (kRun / 8) + t;
+          *reinterpret_cast<uint2*>(dst + e0 + 8 * t) = make_uint2(lo[w], hi[w]);
+        }
+      } else if constexpr (kRun == 4) {  // elements o..o+3 (o = 0 or 4) of a group
+        const int w = run >> 1, h = run & 1;
+        *reinterpret_cast<uint16_t*>(gb + (o >> 1)) = static_cast<uint16_t>(lo[w] >> (16 * h));
+        *reinterpret_cast<uint16_t*>(gb + 4 + (o >> 1)) = static_cast<uint16_t>(hi[w] >> (16 * h));
+      } else {  // kRun == 2: elements o, o+1
+        const int w = run >> 2, q = run & 3;
+        gb[o >> 1] = static_cast<uint8_t>(lo[w] >> (8 * q));
+        gb[4 + (o >> 1)] = static_cast<uint8_t>(hi[w] >> (8 * q));
       }
     }
   }
@@ -335,7 +374,7 @@ cudaError_t launch_t(const RotQuantArgs& a) {
     if (e != cudaSuccess) return e;
   }
   kern<<<grid, tpb, smem, a.stream>>>(reinterpret_cast<const T*>(a.x), a.M, a.K, a.inv_sqrt_b, a.step_scale, a.xq,
-                                      a.xscale, a.xsum, a.mode == 2 ? a.absmax : nullptr);
+                                      a.xscale, a.xsum, a.mode == 2 ? a.absmax : nullptr, a.out_bytes);
   return cudaGetLastError();
 }
 

@@ -39,6 +39,8 @@ SIGNATURES = {
     "qvla_gemm_w4a4": (_I, [_P, _P, _P, _P, _I, _P, _P, _P]),
     "qvla_linear_workspace_bytes": (_S, [_P, _I]),
     "qvla_w4a4_linear": (_I, [_P, _P, _I, _I, _P, _P, _S, _P]),
+    "qvla_linear_quantize": (_I, [_P, _P, _I, _I, _P, _S, _P]),
+    "qvla_linear_gemm": (_I, [_P, _P, _S, _I, _P, _P]),
     "qvla_w4a4_linear_noalloc": (_I, [_P, _P, _I, _I, _P, _P]),
     "qvla_check_device": (_I, [_P]),
 }
@@ -185,6 +187,15 @@ def qvla_linear_workspace_bytes(layer: Layer, M: int) -> int:
 def qvla_w4a4_linear(layer: Layer, x, M: int, step: int, y, workspace, workspace_bytes: int, stream=None) -> None:
     _check(_lib.qvla_w4a4_linear(layer.handle, _ptr(x), M, step, _ptr(y), _ptr(workspace), workspace_bytes,
                                  _stream(stream)))
+
+
+def qvla_linear_quantize(layer: Layer, x, M: int, step: int, workspace, workspace_bytes: int, stream=None) -> None:
+    _check(_lib.qvla_linear_quantize(layer.handle, _ptr(x), M, step, _ptr(workspace), workspace_bytes,
+                                     _stream(stream)))
+
+
+def qvla_linear_gemm(layer: Layer, workspace, workspace_bytes: int, M: int, y, stream=None) -> None:
+    _check(_lib.qvla_linear_gemm(layer.handle, _ptr(workspace), workspace_bytes, M, _ptr(y), _stream(stream)))
 
 
 NOALLOC_SCRATCH_BYTES = 8 << 20

@@ -150,3 +150,19 @@ def test_gated_mlp_block_full_size_sampled():
     G.assert_output_close(y[:, ocols], ref["y"], "bf16")
     layer.close()
     down.close()
+
+
+def test_linear_halves_equal_whole_call():
+    """qvla_linear_quantize + qvla_linear_gemm are the two kernels of qvla_w4a4_linear."""
+    case = W.sweep_linear(300, 2048, 512, seed=31, xdtype="bf16", ydtype="bf16", with_bias=True)
+    layer, _, _ = _layer_from_host_pack(case.w, case.had_block, "bf16", "bf16", bias=case.bias)
+    whole = G.linear(layer, case.x, ydt="bf16")
+    M = case.x.shape[0]
+    nbytes = Q.qvla_linear_workspace_bytes(layer, M)
+    work = torch.empty(nbytes, dtype=torch.uint8, device=G.DEV)
+    y = torch.full((M, layer.N), float("nan"), dtype=torch.bfloat16, device=G.DEV)
+    Q.qvla_linear_quantize(layer, case.x.to(G.DEV), M, -1, work, nbytes, G.stream())
+    Q.qvla_linear_gemm(layer, work, nbytes, M, y, G.stream())
+    Q.qvla_check_device(G.stream())
+    assert np.array_equal(y.double().cpu().numpy(), whole)
+    layer.close()
