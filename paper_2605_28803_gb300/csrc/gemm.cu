@@ -590,7 +590,15 @@ cudaError_t launch_cfg(const GemmArgs& a) {
 template <bool kXBytes, typename OutT>
 cudaError_t launch_out(const GemmArgs& a) {
   if (a.gated) return launch_cfg<256, false, true, kXBytes, OutT>(a);  // gate/up pairs share a 256-row tile
-  if (a.M > 128) return launch_cfg<256, false, false, kXBytes, OutT>(a);
+  if (a.M > 128) {
+    // tile width by estimated time: waves of persistent CTAs x tile width (a narrower tile
+    // wins when the wide one leaves SMs idle, e.g. few output channels and a long K)
+    const long tm = (a.M + kBM - 1) / kBM;
+    const long w256 = (tm * ((a.N + 255) / 256) + a.num_sms - 1) / a.num_sms;
+    const long w128 = (tm * ((a.N + 127) / 128) + a.num_sms - 1) / a.num_sms;
+    if (w128 * 128 < w256 * 256) return launch_cfg<128, false, false, kXBytes, OutT>(a);
+    return launch_cfg<256, false, false, kXBytes, OutT>(a);
+  }
   const int mpad = (a.M + 15) / 16 * 16;
   if (mpad <= 16) return launch_cfg<16, true, false, kXBytes, OutT>(a);
   if (mpad <= 32) return launch_cfg<32, true, false, kXBytes, OutT>(a);
