@@ -161,7 +161,8 @@ qvla_status qvla_rotated_absmax(const void* x, qvla_dtype xdt, int M, int K, int
  * round-to-nearest-even conversion to the layer's output dtype.
  *   xq device [M][K/2], xscale device [M], xsum device [M] (from qvla_rotate_quantize),
  *   y device out [M][N] of the layer's output dtype,
- *   acc device out [M][N] int32, or NULL (debug/test hook: the exact integer accumulator).
+ *   acc device out [M][N] int32, or NULL (debug/test hook: the exact integer accumulator);
+ *       16-byte aligned like xq and y.
  * ------------------------------------------------------------------------------------------ */
 qvla_status qvla_gemm_w4a4(const qvla_layer* layer, const uint8_t* xq, const float* xscale,
                            const int32_t* xsum, int M, void* y, int32_t* acc, void* stream);

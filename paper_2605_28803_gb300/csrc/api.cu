@@ -365,7 +365,8 @@ qvla_status qvla_gemm_w4a4(const qvla_layer* L, const uint8_t* xq, const float* 
   if (qvla_status s = check_rows(M)) return s;
   if (M == 0) return QVLA_OK;
   if (!xq || !xscale || !xsum || !y) return fail(QVLA_ERR_INVALID_ARG, "xq, xscale, xsum and y must not be NULL");
-  if (!aligned16(xq) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "xq and y must be 16-byte aligned");
+  if (!aligned16(xq) || !aligned16(y) || !aligned16(acc))
+    return fail(QVLA_ERR_INVALID_ARG, "xq, y and acc must be 16-byte aligned");
   return launch_gemm(L, xq, 0, xscale, xsum, M, y, acc, stream);
 }
 

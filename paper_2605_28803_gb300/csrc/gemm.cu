@@ -21,7 +21,14 @@
 //
 // Two orientations: for M > 128 the MMA's M side is the activations (tile 128 tokens x 256
 // weight rows); for M <= 128 ("swap") it is the weights (128 weight rows x Mpad tokens),
-// so that a small batch does not waste the 128-row MMA.
+// so that a small batch does not waste the 128-row MMA.  A small batch has few tiles, so in
+// the weight-major orientation a cluster of up to 8 CTAs shares each tile, splitting K: every
+// CTA leaves its FP32 partial (exact, like the whole sum) in its own shared memory and, after
+// a cluster barrier, sums one slice of the tile's rows over the cluster and applies the epilogue.
+//
+// Both kernels of the linear are launched with programmatic stream serialization, so each may
+// start (allocate TMEM, initialise barriers, request weights) while the previous kernel of the
+// stream finishes; everything that touches the previous kernel's data waits for it first.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -29,8 +36,12 @@
 #include <cudaTypedefs.h>
 
 #include <cstdint>
+#include <map>
 #include <mutex>
+#include <set>
+#include <tuple>
 
+#include "griddep.cuh"
 #include "kernels.h"
 #include "ptx.cuh"
 
@@ -79,6 +90,7 @@ struct Params {
   int32_t* acc;
   int M, N;      // N = weight rows of the layer (2H for a gated layer)
   int ldy;       // row length of y (N, or H for a gated layer)
+  int splits;    // weight-major orientation: CTAs of a cluster splitting K (1 = no split)
 };
 
 __device__ __forceinline__ void epi_sync() {
@@ -152,6 +164,22 @@ __device__ __forceinline__ void store_row32(OutT* dst, const uint32_t (&pk)[16],
   }
 }
 
+// Epilogue parameters of 4 consecutive weight rows n .. n + 3 and one token m (split-K reduction);
+// indices past the end are clamped so the loads can be issued unconditionally.
+struct SplitParams {
+  float cm, xs;       // 64 K + 8 xsum[m], xscale[m]
+  float4 wc, ws, bs;  // wcorr, wscale, bias of rows n .. n + 3
+  __device__ __forceinline__ void load(const Params& p, int n, int m) {
+    n = min(n, p.N - 4);
+    m = min(m, p.M - 1);
+    cm = 64.0f * static_cast<float>(p.K) + 8.0f * static_cast<float>(__ldg(p.xsum + m));
+    xs = __ldg(p.xscale + m);
+    wc = __ldg(reinterpret_cast<const float4*>(p.wcorr + n));
+    ws = __ldg(reinterpret_cast<const float4*>(p.wscale + n));
+    bs = __ldg(reinterpret_cast<const float4*>(p.bias + n));
+  }
+};
+
 // kXBytes: the activations arrive as operand bytes ([rows][K], written by the rotate-quantise
 // kernel) and are TMA-loaded with the 128-byte swizzle straight into the MMA operand tile; only
 // the weights are staged and expanded.  Otherwise both operands are packed int4.
@@ -184,7 +212,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   const int tiles_a = (p.rows_a + kBM - 1) / kBM;
   const int tiles_b = (p.rows_b + kBN - 1) / kBN;
   const int ntiles = tiles_a * tiles_b;
-  const int nkb = p.K / kBK;
+  const int nkb_all = p.K / kBK;
+  // split-K (weight-major orientation): the `splits` CTAs of a cluster share one tile, CTA r
+  // taking k-blocks [kb0, kb1); without a split every CTA runs whole tiles persistently
+  const int splits = kSwap ? p.splits : 1;
+  const uint32_t krank = (kSwap && splits > 1) ? cluster_ctarank() : 0u;
+  const int kb0 = (nkb_all * static_cast<int>(krank)) / splits;
+  const int kb1 = (nkb_all * (static_cast<int>(krank) + 1)) / splits;
+  // this CTA's first tile and the tile stride, read where they are used (held in registers
+  // across the role loops they would cost a register in every role)
+#define QVLA_UNIT0 (blockIdx.x / static_cast<unsigned>(splits))
+#define QVLA_NUNITS (gridDim.x / static_cast<unsigned>(splits))
   uint8_t* const raw = smem + C::kStages * C::kStage;  // staging ring after the expanded stages
 
   if (threadIdx.x == 0) {
@@ -207,25 +245,45 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = s_tmem_base;
+  if (threadIdx.x == 0) griddep_launch_dependents();
 
   if (warp == kTmaWarp) {
     // ------------------------------------------------------------------ TMA loads of packed tiles
     if (lane == 0) {
       tma_prefetch_desc(&tmap_a);
       tma_prefetch_desc(&tmap_b);
+      // Weight-major orientation with operand-byte activations: the staging ring holds weights
+      // only, which no earlier kernel writes, so the first stages are requested before waiting
+      // for the previous kernel (a small batch's GEMM is mostly this latency).
+      int pre = 0;
+      if constexpr (kXBytes && kSwap) {
+        const int unit0 = static_cast<int>(QVLA_UNIT0);
+        if (unit0 < ntiles) {
+          const int ta = unit0 % tiles_a;
+          pre = min(C::kStages, kb1 - kb0);
+          for (int i = 0; i < pre; ++i) {
+            const uint32_t bar = smem_u32(&bar_raw_full[i]);
+            mbar_arrive_expect_tx(bar, C::kRaw);
+            tma_load_2d(smem_u32(raw + i * C::kRaw), &tmap_a, (kb0 + i) * (kBK / 2), ta * kBM, bar);
+          }
+        }
+      }
+      griddep_wait();
       int it = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+      for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS) {
         const int ta = tile % tiles_a, tb = tile / tiles_a;
-        for (int kb = 0; kb < nkb; ++kb, ++it) {
+        for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const int s = it % C::kStages;
           const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
-          if (!mbar_wait(smem_u32(&bar_raw_empty[s]), ph ^ 1u)) { ok = false; break; }
-          const uint32_t bar = smem_u32(&bar_raw_full[s]);
-          mbar_arrive_expect_tx(bar, C::kRaw);
-          const uint32_t dst = smem_u32(raw + s * C::kRaw);
-          if constexpr (kStageA) tma_load_2d(dst, &tmap_a, kb * (kBK / 2), ta * kBM, bar);
-          if constexpr (kStageB) tma_load_2d(dst + C::kRawA, &tmap_b, kb * (kBK / 2), tb * kBN, bar);
+          if (it >= pre) {
+            if (!mbar_wait(smem_u32(&bar_raw_empty[s]), ph ^ 1u)) { ok = false; break; }
+            const uint32_t bar = smem_u32(&bar_raw_full[s]);
+            mbar_arrive_expect_tx(bar, C::kRaw);
+            const uint32_t dst = smem_u32(raw + s * C::kRaw);
+            if constexpr (kStageA) tma_load_2d(dst, &tmap_a, kb * (kBK / 2), ta * kBM, bar);
+            if constexpr (kStageB) tma_load_2d(dst + C::kRawA, &tmap_b, kb * (kBK / 2), tb * kBN, bar);
+          }
           if constexpr (kXBytes) {
             // the activation operand goes straight into the expanded stage once the MMAs are done with it
             if (!mbar_wait(smem_u32(&bar_empty[s]), ph ^ 1u)) { ok = false; break; }
@@ -268,8 +326,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     }
     int it = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-      for (int kb = 0; kb < nkb; ++kb, ++it) {
+    for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS) {
+      for (int kb = kb0; kb < kb1; ++kb, ++it) {
         const int s = it % C::kStages;
         const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
         if (!mbar_wait(smem_u32(&bar_raw_full[s]), ph)) { ok = false; break; }
@@ -296,13 +354,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       constexpr uint32_t kIdesc = idesc_e4m3_f32(kBM, kBN);
       int it = 0, tile_iter = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++tile_iter) {
+      for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS, ++tile_iter) {
         const int buf = tile_iter & 1;
         const uint32_t aph = static_cast<uint32_t>(tile_iter >> 1) & 1u;
         if (!mbar_wait(smem_u32(&bar_tempty[buf]), aph ^ 1u)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d = tmem_base + static_cast<uint32_t>(buf * kBN);
-        for (int kb = 0; kb < nkb; ++kb, ++it) {
+        for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const int s = it % C::kStages;
           const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
           if (!mbar_wait(smem_u32(&bar_full[s]), ph)) { ok = false; break; }
@@ -312,7 +370,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
 #pragma unroll
           for (int kk = 0; kk < kBK / 32; ++kk) {
             mma_e4m3(d, smem_desc_sw128(sa + kk * 32), smem_desc_sw128(sb + kk * 32), kIdesc,
-                     (kb | kk) != 0 ? 1u : 0u);
+                     (kb != kb0 || kk != 0) ? 1u : 0u);
           }
           mma_commit(smem_u32(&bar_empty[s]));
         }
@@ -329,7 +387,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     const int et = threadIdx.x;  // 0..127 = TMEM lane
     int tile_iter = 0;
     const float k64 = 64.0f * static_cast<float>(p.K);
-    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++tile_iter) {
+    griddep_wait();  // xscale / xsum come from the previous kernel, and y may still be read by it
+    for (int tile = QVLA_UNIT0; tile < ntiles; tile += QVLA_NUNITS, ++tile_iter) {
       const int ta = tile % tiles_a, tb = tile / tiles_a;
       const int buf = tile_iter & 1;
       const uint32_t aph = static_cast<uint32_t>(tile_iter >> 1) & 1u;
@@ -464,6 +523,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
         const float cn = nok ? __ldg(p.wcorr + n) + k64 : 0.0f;
         const float b = nok ? __ldg(p.bias + n) : 0.0f;
         constexpr int kChunk = kBN < 32 ? kBN : 32;
+        float* part = reinterpret_cast<float*>(smem);  // split-K partial [kBN][128]; the stages are idle now
 #pragma unroll 1
         for (int c0 = 0; c0 < kBN; c0 += kChunk) {
           uint32_t r[32];
@@ -474,6 +534,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
             tmem_ld16(taddr + c0, r);
           }
           tmem_ld_wait();
+          if (splits > 1) {  // leave the partial sums for the cluster reduction below
+#pragma unroll
+            for (int i = 0; i < kChunk; ++i) part[(c0 + i) * kBM + et] = __uint_as_float(r[i]);
+            continue;
+          }
           const int m0 = tb * kBN + c0;
           if (nok) {
 #pragma unroll
@@ -497,8 +562,81 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
 
   tc_fence_before();
   __syncthreads();
+  if constexpr (kSwap) {
+    if (splits > 1) {
+      // split-K: every CTA's partial is in its shared memory; CTA r sums rows
+      // [r R, (r + 1) R) of the tile (R = 128 / splits) over the cluster and applies the
+      // epilogue.  All threads take part; an element is 4 consecutive weight rows of one token
+      // column, and its epilogue parameters are fetched one element ahead (the first while the
+      // cluster barrier completes).
+      cluster_arrive();  // this CTA's partial is published
+      const int R4 = kBM / splits / 4;
+      const int unit0 = static_cast<int>(QVLA_UNIT0);
+      const int total = unit0 < ntiles && !s_epi_abort ? R4 * kBN : 0;
+      const int ta = unit0 % tiles_a, tb = unit0 / tiles_a;
+      auto coords = [&](int e, int& n, int& m, int& row, int& col) {
+        row = (static_cast<int>(krank) * R4 + e % R4) * 4;
+        col = e / R4;
+        n = ta * kBM + row;
+        m = tb * kBN + col;
+      };
+      griddep_wait();
+      SplitParams nxt;
+      int e = threadIdx.x;
+      if (e < total) {
+        int n, m, row, col;
+        coords(e, n, m, row, col);
+        nxt.load(p, n, m);
+      }
+      cluster_wait();
+      const uint32_t part0 = smem_u32(smem);
+      for (; e < total; e += kThreads) {
+        int n, m, row, col;
+        coords(e, n, m, row, col);
+        const SplitParams cur = nxt;
+        if (e + kThreads < total) {
+          int n2, m2, r2, c2;
+          coords(e + kThreads, n2, m2, r2, c2);
+          nxt.load(p, n2, m2);
+        }
+        const uint32_t off = static_cast<uint32_t>((col * kBM + row) * 4);
+        float4 v[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          if (q < splits) v[q] = ld_dsmem_v4(mapa_shared(part0 + off, static_cast<uint32_t>(q)));
+        // exact: the partials add up to the tile's accumulator, an integer below 2^24 times 2^-18
+        float4 sum = v[0];
+#pragma unroll
+        for (int q = 1; q < 8; ++q)
+          if (q < splits) {
+            sum.x += v[q].x;
+            sum.y += v[q].y;
+            sum.z += v[q].z;
+            sum.w += v[q].w;
+          }
+        if (n < p.N && m < p.M) {  // N % 16 == 0, so rows n .. n + 3 all exist
+          const float a0 = fmaf(sum.x, 262144.0f, -(cur.wc.x + cur.cm));
+          const float a1 = fmaf(sum.y, 262144.0f, -(cur.wc.y + cur.cm));
+          const float a2 = fmaf(sum.z, 262144.0f, -(cur.wc.z + cur.cm));
+          const float a3 = fmaf(sum.w, 262144.0f, -(cur.wc.w + cur.cm));
+          const float xs = cur.xs;
+          const uint32_t lo = pack2<OutT>(fmaf(a0, xs * cur.ws.x, cur.bs.x), fmaf(a1, xs * cur.ws.y, cur.bs.y));
+          const uint32_t hi = pack2<OutT>(fmaf(a2, xs * cur.ws.z, cur.bs.z), fmaf(a3, xs * cur.ws.w, cur.bs.w));
+          *reinterpret_cast<uint2*>(reinterpret_cast<OutT*>(p.y) + static_cast<size_t>(m) * p.ldy + n) =
+              make_uint2(lo, hi);
+          if (p.acc)
+            *reinterpret_cast<int4*>(p.acc + static_cast<size_t>(m) * p.N + n) =
+                make_int4(static_cast<int32_t>(a0), static_cast<int32_t>(a1), static_cast<int32_t>(a2),
+                          static_cast<int32_t>(a3));
+        }
+      }
+      cluster_sync();  // no CTA leaves while another still reads its partial
+    }
+  }
   tc_fence_after();
   if (warp == kMmaWarp) tmem_dealloc<C::kTmemCols>(tmem_base);
+#undef QVLA_UNIT0
+#undef QVLA_NUNITS
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
@@ -544,6 +682,40 @@ cudaError_t make_tmap_bytes(CUtensorMap* m, const void* base, int rows, int K, i
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// Raise a kernel's dynamic shared-memory limit, once per kernel and device.
+cudaError_t prepare_kernel(const void* kern, int smem) {
+  static std::mutex mu;
+  static std::set<std::pair<const void*, int>> done;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  if (done.count({kern, dev})) return cudaSuccess;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e == cudaSuccess) done.insert({kern, dev});
+  return e;
+}
+
+// How many clusters of cfg's shape (its only attribute: the cluster dimension) can be resident
+// at once, cached per kernel, cluster size and device; 0 if the query fails.
+int max_active_clusters(const void* kern, const cudaLaunchConfig_t& cfg) {
+  static std::mutex mu;
+  static std::map<std::tuple<const void*, unsigned, int>, int> cache;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  const unsigned cs = cfg.attrs[0].val.clusterDim.x;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find({kern, cs, dev});
+  if (it != cache.end()) return it->second;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    n = 0;
+  }
+  cache[{kern, cs, dev}] = n;
+  return n;
+}
+
 template <int kBN, bool kSwap, bool kGated, bool kXBytes, typename OutT>
 cudaError_t launch_cfg(const GemmArgs& a) {
   constexpr bool kStageA = !(kXBytes && !kSwap);
@@ -573,17 +745,47 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   p.N = a.N;
   p.ldy = a.gated ? a.N / 2 : a.N;
   const int tiles = ((p.rows_a + kBM - 1) / kBM) * ((p.rows_b + kBN - 1) / kBN);
-  const int grid = tiles < a.num_sms ? tiles : a.num_sms;
-  if (grid == 0) return cudaSuccess;
+  if (tiles == 0) return cudaSuccess;
+  auto kern = gemm_w4a4_kernel<kBN, kSwap, kGated, kXBytes, OutT>;
+  cudaError_t e = prepare_kernel(reinterpret_cast<const void*>(kern), C::kSmem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = C::kSmem;
+  cfg.stream = a.stream;
+  // attr[0]: may start while the previous kernel of the stream finishes; attr[1]: cluster shape
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr + 1;
+  cfg.numAttrs = 1;
+  // weight-major orientation: while the tiles alone leave SMs idle, split K over a cluster of
+  // up to 8 CTAs, as long as every cluster of the grid can be resident at once
+  int splits = 1;
+  if (kSwap) {
+    const int nkb = p.K / kBK;
+    while (splits < 8 && 2 * splits <= nkb && tiles * 2 * splits <= a.num_sms) {
+      attr[1].val.clusterDim.x = static_cast<unsigned>(2 * splits);
+      cfg.gridDim = dim3(tiles * 2 * splits);
+      if (max_active_clusters(reinterpret_cast<const void*>(kern), cfg) < tiles) break;
+      splits *= 2;
+    }
+  }
+  p.splits = splits;
+  attr[1].val.clusterDim.x = static_cast<unsigned>(splits);
+  cfg.gridDim = dim3(splits > 1 ? tiles * splits : (tiles < a.num_sms ? tiles : a.num_sms));
+  cfg.attrs = attr;
+  cfg.numAttrs = splits > 1 ? 2 : 1;  // a cluster launch only when K is split
   CUtensorMap ta, tb;
-  cudaError_t e = kStageA ? make_tmap(&ta, p.a, p.rows_a, p.K / 2, kBM) : make_tmap_bytes(&ta, p.a, p.rows_a, p.K, kBM);
+  e = kStageA ? make_tmap(&ta, p.a, p.rows_a, p.K / 2, kBM) : make_tmap_bytes(&ta, p.a, p.rows_a, p.K, kBM);
   if (e == cudaSuccess)
     e = kStageB ? make_tmap(&tb, p.b, p.rows_b, p.K / 2, kBN) : make_tmap_bytes(&tb, p.b, p.rows_b, p.K, kBN);
   if (e != cudaSuccess) return e;
-  auto kern = gemm_w4a4_kernel<kBN, kSwap, kGated, kXBytes, OutT>;
-  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+  e = cudaLaunchKernelEx(&cfg, kern, ta, tb, p);
   if (e != cudaSuccess) return e;
-  kern<<<grid, kThreads, C::kSmem, a.stream>>>(ta, tb, p);
   return cudaGetLastError();
 }
 

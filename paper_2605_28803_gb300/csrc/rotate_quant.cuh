@@ -15,8 +15,10 @@
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstdint>
 
+#include "griddep.cuh"
 #include "kernels.h"
 
 namespace qvla {
@@ -165,6 +167,8 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
     s_sum[tid] = 0u;
   }
 
+  griddep_wait();  // x comes from the previous kernel, which may still read xq / xscale / xsum
+  griddep_launch_dependents();
   float2 v[kN];
   if (active) {
     const T* src = x + static_cast<size_t>(m) * K + static_cast<size_t>(j) * kEpt;
@@ -370,11 +374,31 @@ cudaError_t launch_t(const RotQuantArgs& a) {
   const size_t smem = (kLogB > ((kEpt == 128) ? 7 : 6)) ? static_cast<size_t>(tpb) * kEpt * sizeof(float) : 0;
   auto kern = rotate_quant_kernel<T, kLogB, kEpt, kStep>;
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    // raise the shared-memory limit once per device (bit d of the mask)
+    static std::atomic<unsigned long long> raised{0};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
+    const unsigned long long bit = 1ull << (dev & 63);
+    if (!(raised.load() & bit)) {
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+      if (e != cudaSuccess) return e;
+      raised.fetch_or(bit);
+    }
   }
-  kern<<<grid, tpb, smem, a.stream>>>(reinterpret_cast<const T*>(a.x), a.M, a.K, a.inv_sqrt_b, a.step_scale, a.xq,
-                                      a.xscale, a.xsum, a.mode == 2 ? a.absmax : nullptr, a.out_bytes);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(tpb);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = a.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // may overlap the previous kernel
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kern, reinterpret_cast<const T*>(a.x), a.M, a.K, a.inv_sqrt_b, a.step_scale,
+                                     a.xq, a.xscale, a.xsum, a.mode == 2 ? a.absmax : nullptr, a.out_bytes);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

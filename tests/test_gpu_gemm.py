@@ -1,7 +1,8 @@
 """GPU parity of the int4 x int4 GEMM and its dequantisation epilogue (Sec. 4.2, Eq. 7).
 
 G2: on the oracle's codes the int32 accumulator is bit-exact for every tile shape, ragged M and
-N edges and both orientations (tokens on the MMA's M side for M > 128, weights otherwise).
+N edges and both orientations (tokens on the MMA's M side for M > 128, weights otherwise),
+including the weight-major split of K over clusters of 2, 4 and 8 CTAs.
 G3: the E4M3 / FP32 tensor-core path stays exact at the largest sums K = 16384 allows.
 G5: outputs within 2e-3 of the tensor's maximum magnitude."""
 
@@ -37,6 +38,9 @@ def _run(M, N, K, seed, ydt="f16", with_bias=True):
     (1, 16, 128), (5, 48, 512), (16, 256, 2048), (17, 272, 1024), (50, 1024, 1024), (64, 4096, 1024),
     (100, 512, 4096), (128, 1024, 512), (129, 256, 512), (256, 512, 2048), (300, 272, 1024), (816, 1024, 2048),
     (816, 2048, 16384), (1000, 2048, 128),
+    # weight-major split-K: a cluster of 2 with several reduction elements per thread, 5
+    # k-blocks over 4 CTAs (uneven slices) with a ragged weight tile, a decode row at K = 16384
+    (100, 8192, 1024), (33, 400, 640), (1, 2048, 16384),
 ])
 def test_gemm_accumulator_bit_exact(M, N, K):
     acc, ref_acc, y, ref_y = _run(M, N, K, seed=M * 7 + N + K)

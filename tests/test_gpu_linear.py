@@ -44,7 +44,8 @@ def test_single_layer_per_step_table_all_steps():
 
 
 @pytest.mark.parametrize("M,K,N", [(1, 1024, 1024), (16, 2048, 2048), (50, 1024, 4096), (256, 2048, 2048),
-                                   (816, 2048, 1024), (300, 16384, 2048), (3200, 1024, 1024)])
+                                   (816, 2048, 1024), (300, 16384, 2048), (3200, 1024, 1024),
+                                   (1, 16384, 2048), (100, 1024, 8192), (50, 4096, 1024)])
 def test_linear_per_token_sweep_points(M, K, N):
     case = W.sweep_linear(M, K, N, xdtype="bf16", ydtype="bf16", with_bias=True)
     layer, wq, ws = _layer_from_host_pack(case.w, case.had_block, "bf16", "bf16", bias=case.bias)
