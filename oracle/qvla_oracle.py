@@ -41,6 +41,7 @@ pinned by closed forms, invariants, library special cases and brute force in
 
 from __future__ import annotations
 
+import functools
 import math
 
 import numpy as np
@@ -70,8 +71,16 @@ def sylvester_hadamard(n: int) -> np.ndarray:
 
 
 def normalized_hadamard(n: int) -> np.ndarray:
-    """H / sqrt(n) in float64: the orthogonal matrix of Sec. 4.1 / Eq. 3."""
-    return sylvester_hadamard(n).astype(np.float64) / math.sqrt(n)
+    """H / sqrt(n) in float64: the orthogonal matrix of Sec. 4.1 / Eq. 3.  Built once per
+    order and returned read-only (the stacks rotate thousands of rows with the same H)."""
+    return _normalized_hadamard_cached(n)
+
+
+@functools.lru_cache(maxsize=8)
+def _normalized_hadamard_cached(n: int) -> np.ndarray:
+    h = sylvester_hadamard(n).astype(np.float64) / math.sqrt(n)
+    h.setflags(write=False)
+    return h
 
 
 def block_hadamard_rotate(x: np.ndarray, had_block: int) -> np.ndarray:

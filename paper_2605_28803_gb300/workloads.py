@@ -168,3 +168,115 @@ DIT_LAYER_SHAPES = (("q", 1024, 1024), ("k", 1024, 1024), ("v", 1024, 1024), ("o
 BACKBONE_LAYER_SHAPES = (("q", 2048, 2048), ("k", 2048, 256), ("v", 2048, 256), ("o", 2048, 2048),
                          ("gate", 2048, 16384), ("up", 2048, 16384), ("down", 16384, 2048))
 """(name, K, N) of one backbone decoder layer (Gemma-2B-like, 18 layers)."""
+
+
+# --------------------------------------------------------------------------------------
+# Layer stacks: pre-rotated, pre-quantised weights drawn directly as int4 codes
+# --------------------------------------------------------------------------------------
+
+def pack_nibbles(codes: np.ndarray) -> np.ndarray:
+    """int8 codes [..., K] in [-8, 7] -> the packed storage layout (byte j: code 2j in the low
+    nibble, code 2j+1 in the high nibble, 4-bit two's complement), uint8 [..., K/2]."""
+    u = (np.asarray(codes).astype(np.int16) & 0xF).astype(np.uint8)
+    return np.ascontiguousarray(u[..., 0::2] | (u[..., 1::2] << 4))
+
+
+@dataclass
+class StackWeights:
+    """One linear of a stack: its weights as int4 codes (what the offline fold and quantiser
+    would produce) with per-output-channel scales.  For a gated layer the rows are the H gate
+    rows, then the H up rows."""
+    name: str
+    k: int
+    n: int                    # output features (H for a gated layer)
+    had_block: int
+    packed: np.ndarray        # uint8 [rows, k/2]
+    wscale: np.ndarray        # float32 [rows]
+    bias: np.ndarray | None   # float32 [rows] or None
+    gated: bool = False
+    codes: np.ndarray | None = None  # int8 [rows, k] when drawn as codes
+
+    def weight_codes(self) -> np.ndarray:
+        """int8 codes [rows, k], unpacked from the storage layout when not kept."""
+        if self.codes is not None:
+            return self.codes
+        b = self.packed
+        out = np.empty(b.shape[:-1] + (b.shape[-1] * 2,), dtype=np.int8)
+        lo = (b & 0xF).astype(np.int16)
+        hi = (b >> 4).astype(np.int16)
+        out[..., 0::2] = np.where(lo > 7, lo - 16, lo)
+        out[..., 1::2] = np.where(hi > 7, hi - 16, hi)
+        return out
+
+
+def gaussian_codes(rng, rows: int, k: int, sigma: float = 2.0) -> np.ndarray:
+    """Weight codes shaped like per-channel int4 codes of Gaussian weights: N(0, sigma^2)
+    rounded to integers and clipped to [-7, 7], int8 [rows, k]."""
+    return np.clip(np.rint(rng.standard_normal((rows, k), dtype=np.float32) * np.float32(sigma)), -7, 7).astype(np.int8)
+
+
+def _weight_scales(rng, rows: int, k: int) -> np.ndarray:
+    """Per-channel scales of weights ~ N(0, 1/K): about max|w| / 7 ~ 0.5 / sqrt(K), +-20%."""
+    return (rng.uniform(0.8, 1.2, rows) * 0.5 / np.sqrt(k)).astype(np.float32)
+
+
+DIT_STACK_LAYERS = (("qkv", 1024, 3072), ("o", 1024, 1024), ("up", 1024, 4096), ("down", 4096, 1024))
+"""(name, K, N) of one DiT block as run: Q, K and V read the same input with the same per-step
+table, so they form one 1024 -> 3072 linear whose output columns are [Q | K | V]."""
+
+
+def dit_stack(seed: int = 2, layers: int = 18) -> list:
+    """Weights of the DiT action head's 18 blocks: per block qkv 1024 -> 3072, o 1024 -> 1024,
+    up 1024 -> 4096, down 4096 -> 1024, Hadamard block = K, with biases.  Codes ~ rounded
+    N(0, 2^2) in [-7, 7].  Draw order per layer and linear: codes, scales, bias."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for layer in range(layers):
+        for name, k, n in DIT_STACK_LAYERS:
+            codes = gaussian_codes(rng, n, k)
+            ws = _weight_scales(rng, n, k)
+            bias = (rng.standard_normal(n, dtype=np.float32) * np.float32(0.05)).astype(np.float32)
+            out.append(StackWeights(f"{layer}.{name}", k, n, k, pack_nibbles(codes), ws, bias, codes=codes))
+    return out
+
+
+def dit_layer_input(seed: int, index: int, t: int, m: int, k: int, steps: int = 10) -> np.ndarray:
+    """Input of linear `index` of the DiT stack at denoising step t: N(0, sigma_t^2) [m, k]
+    float32 with sigma_t drifting from 4.0 (t = 0) to 0.5 (t = T-1).  Each (index, t) has its
+    own stream, so any subset can be drawn."""
+    rng = np.random.default_rng([seed, index, t])
+    return rng.standard_normal((m, k), dtype=np.float32) * np.float32(dit_input_std(t, steps))
+
+
+BACKBONE_STACK_LAYERS = (("qkv", 2048, 2560, False), ("o", 2048, 2048, False), ("gate_up", 2048, 16384, True),
+                         ("down", 16384, 2048, False))
+"""(name, K, N, gated) of one backbone layer as run: Q (2048) and K/V (256 each) share their
+input and form one 2048 -> 2560 linear; gate and up (2048 -> 16384 each) form one gated layer
+whose output is gelu(gate) * up."""
+
+
+def backbone_stack(seed: int = 3, layers: int = 18, had_wide: int = 2048) -> list:
+    """Weights of the 18-layer backbone (hidden 2048, MLP 16384): 1.98 G int4 codes drawn as
+    uniform random bytes (codes uniform in [-8, 7]; the packed format carries -8), with
+    per-channel scales and no bias.  Hadamard block = K for K = 2048, 8 x 2048 blocks for
+    K = 16384.  Draw order per layer and linear: bytes, scales."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for layer in range(layers):
+        for name, k, n, gated in BACKBONE_STACK_LAYERS:
+            rows = 2 * n if gated else n
+            packed = rng.integers(0, 256, (rows, k // 2), dtype=np.uint8)
+            ws = _weight_scales(rng, rows, k)
+            out.append(StackWeights(f"{layer}.{name}", k, n, min(k, had_wide), packed, ws, None, gated=gated))
+    return out
+
+
+def backbone_layer_input(seed: int, index: int, m: int, k: int, frac: float = 0.002, factor: float = 20.0) -> np.ndarray:
+    """Input of linear `index` of the backbone stack: N(0, 1) [m, k] float32 with a fixed 0.2%
+    of channels (per linear) scaled x20."""
+    rng = np.random.default_rng([seed, index])
+    n_out = max(1, int(round(frac * k)))
+    idx = rng.choice(k, n_out, replace=False)
+    x = rng.standard_normal((m, k), dtype=np.float32)
+    x[:, idx] *= np.float32(factor)
+    return x

@@ -422,8 +422,11 @@ MUTANTS = {
 
 
 @pytest.mark.parametrize("name", sorted(MUTANTS))
-def test_mutants(name, monkeypatch):
+def test_mutants(name, monkeypatch, request):
     attr, fn = MUTANTS[name]
+    # the normalised Hadamard is cached: rebuild it from the mutant, and again after it is undone
+    O._normalized_hadamard_cached.cache_clear()
+    request.addfinalizer(O._normalized_hadamard_cached.cache_clear)
     monkeypatch.setattr(O, attr, fn)
     failed = []
     for pin_name, pin in PINS.items():
