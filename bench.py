@@ -13,6 +13,13 @@ Student-t channels, Gaussian weights) in the shapes of the Pi-0.5 backbone MLP.
 
 Prints one JSON line (rank 0).  Under torchrun each rank runs its own replica of the block
 (weak scaling, no collective on the data path); the time is the maximum over ranks.
+
+The line also carries the two layer stacks (skipped with --no-stacks):
+  "dit": the DiT action head, 18 blocks (qkv 1024 -> 3072, o 1024 -> 1024, up 1024 -> 4096,
+         down 4096 -> 1024) at M = 50 tokens with per-step scale tables, one CUDA graph per
+         denoising step: microseconds per step (L2 flushed before each) and per 10-step rollout;
+  "backbone": 18 layers of hidden 2048 with the gated 16384 MLP, per-token scales, one forward
+         pass at M = 816 (TOPS) and at M = 1 (HBM-bound: GB/s of packed weights).
 """
 
 from __future__ import annotations
@@ -51,6 +58,7 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--sets", type=int, default=3, help="rotating weight+activation sets (working set > L2)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="CPU-baseline sample budget")
+    ap.add_argument("--no-stacks", action="store_true", help="skip the DiT and backbone stack legs")
     return ap.parse_args()
 
 
@@ -224,7 +232,10 @@ def run_ours(args):
 
     # ---- device-timed region: inputs resident in HBM ----
     K = args.steps
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    # per-kernel events on every EVERY-th step only: between events the kernels of the other
+    # steps keep overlapping their launch with the previous kernel's tail
+    EVERY = 8
+    evs = {i: [torch.cuda.Event(enable_timing=True) for _ in range(5)] for i in range(0, K, EVERY)}
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
     barrier(world)
@@ -232,17 +243,18 @@ def run_ours(args):
     clocks.start()
     t0.record(stream)
     for i in range(K):
-        step(sets[i % args.sets], evs[i])
+        step(sets[i % args.sets], evs.get(i))
     t1.record(stream)
     torch.cuda.synchronize()
     barrier(world)
     clk = clocks.stop()
     Q.qvla_check_device(stream)
     ms = max_over_ranks(world, t0.elapsed_time(t1), dev)
-    rqx_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / K
-    gemm_gu_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / K
-    rqh_ms = sum(e[2].elapsed_time(e[3]) for e in evs) / K
-    gemm_dn_ms = sum(e[3].elapsed_time(e[4]) for e in evs) / K
+    ne = len(evs)
+    rqx_ms = sum(e[0].elapsed_time(e[1]) for e in evs.values()) / ne
+    gemm_gu_ms = sum(e[1].elapsed_time(e[2]) for e in evs.values()) / ne
+    rqh_ms = sum(e[2].elapsed_time(e[3]) for e in evs.values()) / ne
+    gemm_dn_ms = sum(e[3].elapsed_time(e[4]) for e in evs.values()) / ne
     value = world * OPS_STEP * K / (ms * 1e-3) / 1e12
 
     # ---- end to end through the public API with host buffers ----
@@ -266,7 +278,8 @@ def run_ours(args):
     ms2 = max_over_ranks(world, e0.elapsed_time(e1), dev)
     e2e = world * OPS_STEP * K2 / (ms2 * 1e-3) / 1e12
 
-    peak_tflops, _, peak_src = peaks()
+    peak_tflops, peak_gbs, peak_src = peaks()
+    stacks = None if args.no_stacks else run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src)
     achieved = (OPS_GATEUP + OPS_DOWN) / ((gemm_gu_ms + gemm_dn_ms) * 1e-3) / 1e12
     cpu = cpu_baseline(mlp, packed, args.cpu_seconds) if (rank == 0 and world == 1) else None
     if rank == 0:
@@ -281,6 +294,7 @@ def run_ours(args):
                          "unit": "TFLOP/s", "frac": round(achieved / peak_tflops, 4), "traffic": gemm_traffic(),
                          "kernel": "gemm_w4a4 (gate/up + down launches)",
                          "peak_note": f"{peak_src} sustained bf16 x {FP8_OVER_BF16:g} (nominal E4M3/bf16 ratio)"},
+            "kernels_us_note": f"CUDA events around each launch on every {EVERY}th timed step",
             "kernels_us": {"rotate_quantize_x": round(rqx_ms * 1e3, 2), "gemm_gate_up": round(gemm_gu_ms * 1e3, 2),
                            "rotate_quantize_h": round(rqh_ms * 1e3, 2), "gemm_down": round(gemm_dn_ms * 1e3, 2)},
             "e2e": {"value": round(e2e, 2), "unit": "TOPS", "h2d_bytes_per_step": M * K_IN * 2,
@@ -289,10 +303,128 @@ def run_ours(args):
             "clocks": clk,
             "cpu_baseline": cpu,
         }
+        if stacks:
+            line.update(stacks)
         print(json.dumps(line), flush=True)
     for s in sets:
         s["gu"].close()
         s["dn"].close()
+
+
+# --------------------------------------------------------------------------------------
+# the layer stacks
+# --------------------------------------------------------------------------------------
+
+DIT_SEED, DIT_M, DIT_T, DIT_CAL_ROWS = 2, 50, 10, 16
+
+
+def _algorithmic_bytes(weights, m, xb=2, yb=2):
+    """Bytes a fused linear must move: activations in, packed weights, scales and bias, outputs."""
+    return sum(xb * m * w.k + w.packed.nbytes + 8 * w.packed.shape[0] + yb * m * w.n for w in weights)
+
+
+def _time_replays(fn, reps, flush=None, stream=None):
+    """Mean milliseconds of fn() over reps runs, each bracketed by CUDA events on the launching
+    stream; flush() (outside the events) runs first when given."""
+    evs = []
+    for _ in range(reps):
+        if flush is not None:
+            flush()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        evs.append((a, b))
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in evs) / reps
+
+
+def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
+    from paper_2605_28803_gb300 import qvla as Q
+    from paper_2605_28803_gb300 import stack as S
+    from paper_2605_28803_gb300 import workloads as W
+
+    scratch = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # 256 MB > 129 MB L2
+
+    def flush():
+        scratch.zero_()
+
+    # ---- DiT action head: per-step tables calibrated with the library's rotated-absmax pass ----
+    weights = W.dit_stack(DIT_SEED)
+    st = S.LinearStack(weights, DIT_M, "f16", "f16", dev, input_sets=DIT_T)
+    peak = torch.zeros(1, dtype=torch.float32, device=dev)
+    tables = []
+    for i, w in enumerate(weights):
+        tab = []
+        for t in range(DIT_T):
+            xc = torch.from_numpy(W.dit_layer_input(DIT_SEED + 1000, i, t, DIT_CAL_ROWS, w.k, DIT_T)).to(dev, torch.float16)
+            peak.zero_()
+            Q.qvla_rotated_absmax(xc, Q.F16, DIT_CAL_ROWS, w.k, w.had_block, peak, stream)
+            tab.append(np.float32(peak.item()) / np.float32(7))
+        tables.append(np.asarray(tab, dtype=np.float32))
+        for t in range(DIT_T):
+            st.set_input(i, torch.from_numpy(W.dit_layer_input(DIT_SEED, i, t, DIT_M, w.k, DIT_T)), t)
+    st.set_step_tables(tables)
+    graphs = [st.capture(t) for t in range(DIT_T)]
+    for _ in range(3):
+        for g in graphs:
+            g.replay()
+    torch.cuda.synchronize()
+    Q.qvla_check_device(stream)
+    reps = 20
+    step_ms = sum(_time_replays(g.replay, reps, flush, stream) for g in graphs) / DIT_T
+    roll_ms = _time_replays(lambda: [g.replay() for g in graphs], reps, flush, stream)
+    warm_ms = _time_replays(lambda: [g.replay() for g in graphs], reps, None, stream) / DIT_T
+    Q.qvla_check_device(stream)
+    dit_bytes = _algorithmic_bytes(weights, DIT_M)
+    dit_gbs = dit_bytes / (step_ms * 1e-3) / 1e9
+    dit = {
+        "us_per_step": round(step_ms * 1e3, 2), "us_per_rollout": round(roll_ms * 1e3, 2),
+        "us_per_step_warm": round(warm_ms * 1e3, 2), "steps": DIT_T, "tokens": DIT_M,
+        "linears_per_step": len(weights), "gpu_launches_per_step": 2 * len(weights),
+        "weight_bytes": st.weight_bytes, "ops_per_step": st.ops,
+        "roofline": {"bound": "hbm", "achieved": round(dit_gbs, 1), "peak": round(peak_gbs, 1), "unit": "GB/s",
+                     "frac": round(dit_gbs / peak_gbs, 4), "bytes_per_step": dit_bytes,
+                     "peak_note": f"{peak_src} HBM copy bandwidth"},
+        "timing": "CUDA-graph replay per step, L2 flushed (256 MB write) before each timed step or rollout; "
+                  "'warm' = 10 steps back to back without a flush",
+        "tables": "per-step, per-layer, calibrated with qvla_rotated_absmax on a separate 16-token draw",
+    }
+    st.close()
+    del graphs, st
+    torch.cuda.empty_cache()
+
+    # ---- backbone forward at M = 816 and M = 1 (per-token scales) ----
+    weights = W.backbone_stack(seed=3)
+    bb = {"layers": 18, "linears": len(weights), "weight_bytes": int(sum(w.packed.nbytes for w in weights))}
+    for m in (816, 1):
+        st = S.LinearStack(weights, m, "bf16", "bf16", dev)
+        for i, w in enumerate(weights):
+            st.set_input(i, torch.from_numpy(W.backbone_layer_input(3, i, m, w.k)))
+        g = st.capture(-1)
+        g.replay()
+        torch.cuda.synchronize()
+        Q.qvla_check_device(stream)
+        ms = _time_replays(g.replay, 10, flush, stream)
+        Q.qvla_check_device(stream)
+        if m > 1:
+            tops = st.ops / (ms * 1e-3) / 1e12
+            bb["m816"] = {"us_per_forward": round(ms * 1e3, 1), "tops": round(tops, 1),
+                          "roofline": {"bound": "tensor", "achieved": round(tops, 1), "peak": round(peak_tflops, 1),
+                                       "unit": "TFLOP/s", "frac": round(tops / peak_tflops, 4)}}
+        else:
+            nbytes = _algorithmic_bytes(weights, m)
+            gbs = nbytes / (ms * 1e-3) / 1e9
+            bb["m1"] = {"us_per_forward": round(ms * 1e3, 1),
+                        "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": round(peak_gbs, 1),
+                                     "unit": "GB/s", "frac": round(gbs / peak_gbs, 4), "bytes": nbytes}}
+        st.close()
+        del g, st
+        torch.cuda.empty_cache()
+    bb["timing"] = "CUDA-graph replay of one forward (2 kernels per linear), L2 flushed before each"
+    del scratch
+    torch.cuda.empty_cache()
+    return {"dit": dit, "backbone": bb}
 
 
 # --------------------------------------------------------------------------------------

@@ -19,7 +19,7 @@ struct qvla_layer {
   int gated = 0;
   int xdt = 0, ydt = 0;
   int device = 0;
-  uint8_t* wq = nullptr;      // device [N][K/2]
+  uint8_t* wq = nullptr;      // device, tiled: [groups][K/128][128 rows][64 B] (see upload_layer)
   float* wscale = nullptr;    // device [N]
   float* wcorr = nullptr;     // device [N]: 8 * (sum of the codes of row n), the GEMM's offset correction
   float* bias = nullptr;      // device [N] (zeros when the layer was given none)
@@ -176,12 +176,29 @@ static qvla_status upload_layer(int N, int K, int had_block, qvla_dtype xdt, qvl
   L->xdt = xdt;
   L->ydt = ydt;
   cudaGetDevice(&L->device);
-  const size_t wbytes = static_cast<size_t>(N) * (K / 2);
+  // Weights are stored tiled: each group of 128 rows x one k-block of 128 codes (64 bytes per
+  // row) is one contiguous 8 KB chunk, chunks ordered by row group, then k-block; rows past N
+  // are zero, and the number of groups is even (a 256-row GEMM tile reads groups in pairs).
+  // The GEMM fetches a chunk with one bulk copy instead of 128 separate 64-byte rows.
+  const int groups = ((N + 255) / 256) * 2, kblocks = K / 128;
+  const size_t rb = static_cast<size_t>(K / 2);
+  const size_t wbytes = static_cast<size_t>(groups) * kblocks * 8192;
+  std::vector<uint8_t> tiled;
+  try {
+    tiled.assign(wbytes, 0);
+  } catch (...) {
+    delete L;
+    return fail(QVLA_ERR_OOM, "host allocation failed");
+  }
+  for (int n = 0; n < N; ++n)
+    for (int kb = 0; kb < kblocks; ++kb)
+      std::memcpy(tiled.data() + ((static_cast<size_t>(n / 128) * kblocks + kb) * 128 + n % 128) * 64,
+                  wq + n * rb + static_cast<size_t>(kb) * 64, 64);
   cudaError_t e = cudaMalloc(&L->wq, wbytes);
   if (e == cudaSuccess) e = cudaMalloc(&L->wscale, N * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&L->wcorr, N * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&L->bias, N * sizeof(float));
-  if (e == cudaSuccess) e = cudaMemcpy(L->wq, wq, wbytes, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(L->wq, tiled.data(), wbytes, cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(L->wscale, wscale, N * sizeof(float), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(L->wcorr, wcorr.data(), N * sizeof(float), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(L->bias, bias, N * sizeof(float), cudaMemcpyHostToDevice);

@@ -78,8 +78,11 @@ struct Cfg {
 };
 
 struct Params {
-  const uint8_t* a;   // MMA A operand rows [rows_a][K/2]
-  const uint8_t* b;   // MMA B operand rows [rows_b][K/2]
+  // The MMA operands: the weights (A when swapped, else B) in the layer's tiled layout, one
+  // contiguous 8 KB chunk per 128 rows x k-block ([rows/128][K/128][128][64 B]); the
+  // activations through a tensor map.
+  const uint8_t* a;
+  const uint8_t* b;
   int rows_a, rows_b, K;
   const float* xscale;
   const int32_t* xsum;
@@ -189,6 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   constexpr bool kStageA = !(kXBytes && !kSwap);  // operand A is the activations unless swapped
   constexpr bool kStageB = !(kXBytes && kSwap);
   using C = Cfg<kBN, kStageA, kStageB>;
+  static_assert(kSwap || kBN % 128 == 0, "a weight tile is whole 128-row chunks");
   extern __shared__ uint8_t dyn_smem[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~uintptr_t(1023));
 
@@ -250,8 +254,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   if (warp == kTmaWarp) {
     // ------------------------------------------------------------------ TMA loads of packed tiles
     if (lane == 0) {
-      tma_prefetch_desc(&tmap_a);
-      tma_prefetch_desc(&tmap_b);
+      tma_prefetch_desc(kSwap ? &tmap_b : &tmap_a);  // the activations' map (the weights need none)
       // Weight-major orientation with operand-byte activations: the staging ring holds weights
       // only, which no earlier kernel writes, so the first stages are requested before waiting
       // for the previous kernel (a small batch's GEMM is mostly this latency).
@@ -264,7 +267,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
           for (int i = 0; i < pre; ++i) {
             const uint32_t bar = smem_u32(&bar_raw_full[i]);
             mbar_arrive_expect_tx(bar, C::kRaw);
-            tma_load_2d(smem_u32(raw + i * C::kRaw), &tmap_a, (kb0 + i) * (kBK / 2), ta * kBM, bar);
+            bulk_load(smem_u32(raw + i * C::kRaw), p.a + (static_cast<size_t>(ta) * nkb_all + kb0 + i) * 8192, 8192, bar);
           }
         }
       }
@@ -281,8 +284,23 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
             const uint32_t bar = smem_u32(&bar_raw_full[s]);
             mbar_arrive_expect_tx(bar, C::kRaw);
             const uint32_t dst = smem_u32(raw + s * C::kRaw);
-            if constexpr (kStageA) tma_load_2d(dst, &tmap_a, kb * (kBK / 2), ta * kBM, bar);
-            if constexpr (kStageB) tma_load_2d(dst + C::kRawA, &tmap_b, kb * (kBK / 2), tb * kBN, bar);
+            if constexpr (kStageA) {
+              if constexpr (kSwap) {
+                bulk_load(dst, p.a + (static_cast<size_t>(ta) * nkb_all + kb) * 8192, 8192, bar);
+              } else {
+                tma_load_2d(dst, &tmap_a, kb * (kBK / 2), ta * kBM, bar);
+              }
+            }
+            if constexpr (kStageB) {
+              if constexpr (!kSwap) {
+#pragma unroll
+                for (int c = 0; c < kBN / 128; ++c)
+                  bulk_load(dst + C::kRawA + c * 8192,
+                            p.b + (static_cast<size_t>(tb * (kBN / 128) + c) * nkb_all + kb) * 8192, 8192, bar);
+              } else {
+                tma_load_2d(dst + C::kRawA, &tmap_b, kb * (kBK / 2), tb * kBN, bar);
+              }
+            }
           }
           if constexpr (kXBytes) {
             // the activation operand goes straight into the expanded stage once the MMAs are done with it
@@ -779,10 +797,13 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   cfg.gridDim = dim3(splits > 1 ? tiles * splits : (tiles < a.num_sms ? tiles : a.num_sms));
   cfg.attrs = attr;
   cfg.numAttrs = splits > 1 ? 2 : 1;  // a cluster launch only when K is split
-  CUtensorMap ta, tb;
-  e = kStageA ? make_tmap(&ta, p.a, p.rows_a, p.K / 2, kBM) : make_tmap_bytes(&ta, p.a, p.rows_a, p.K, kBM);
-  if (e == cudaSuccess)
+  // a tensor map for the activations only (the weights arrive as contiguous chunks)
+  CUtensorMap ta = {}, tb = {};
+  if constexpr (kSwap) {
     e = kStageB ? make_tmap(&tb, p.b, p.rows_b, p.K / 2, kBN) : make_tmap_bytes(&tb, p.b, p.rows_b, p.K, kBN);
+  } else {
+    e = kStageA ? make_tmap(&ta, p.a, p.rows_a, p.K / 2, kBM) : make_tmap_bytes(&ta, p.a, p.rows_a, p.K, kBM);
+  }
   if (e != cudaSuccess) return e;
   e = cudaLaunchKernelEx(&cfg, kern, ta, tb, p);
   if (e != cudaSuccess) return e;

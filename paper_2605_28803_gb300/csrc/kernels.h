@@ -33,7 +33,8 @@ struct GemmArgs {
   int x_bytes;             // 1: xq holds the rotate-quantise kernel's operand bytes
   const float* xscale;     // device [M]
   const int32_t* xsum;     // device [M]
-  const uint8_t* wq;       // device [N][K/2] weight codes
+  const uint8_t* wq;       // device weight codes, tiled: 8 KB chunks of 128 rows x 128 codes,
+                           // [groups][K/128][128][64 B], groups even (rows past N are zero)
   const float* wscale;     // device [N]
   const float* wcorr;      // device [N]: 8 * sum_k wq[n,k] as float
   const float* bias;       // device [N] (zeros when the layer has no bias)

@@ -8,8 +8,10 @@ consecutive launches overlap their set-up with the previous kernel's tail; ``cap
 a whole pass as a CUDA graph, which removes the host launch cost as well.  The per-step scale
 of a DiT layer is fixed at launch, so a DiT stack has one graph per denoising step.
 
-One workspace (the largest any layer needs) serves all layers: the linears run in stream order
-and each kernel waits for its predecessor before touching the workspace.
+A stack may hold several input sets (one per denoising step, say): a pass at step t reads set
+t when there are as many sets as steps.  One workspace (the largest any layer needs) serves all
+layers: the linears run in stream order and each kernel waits for its predecessor before
+touching the workspace.
 """
 
 from __future__ import annotations
@@ -26,12 +28,13 @@ class LinearStack:
     """Layers built from ``workloads.StackWeights``-like records (fields name, k, n,
     had_block, packed, wscale, bias, gated), all with m rows of input."""
 
-    def __init__(self, weights, m: int, xdtype: str = "f16", ydtype: str = "f16", device=None):
+    def __init__(self, weights, m: int, xdtype: str = "f16", ydtype: str = "f16", device=None, input_sets: int = 1):
         self.m = m
         self.device = torch.device("cuda") if device is None else device
         xdt, self.xtorch = _DT[xdtype]
         ydt, self.ytorch = _DT[ydtype]
-        self.layers, self.names, self.x, self.y = [], [], [], []
+        self.layers, self.names, self.y = [], [], []
+        self.sets = [[] for _ in range(input_sets)]
         for w in weights:
             if w.gated:
                 h = w.n
@@ -43,7 +46,8 @@ class LinearStack:
                 layer = Q.qvla_layer_create(w.n, w.k, w.had_block, xdt, ydt, w.packed, w.wscale, w.bias)
             self.layers.append(layer)
             self.names.append(w.name)
-            self.x.append(torch.zeros(m, w.k, dtype=self.xtorch, device=self.device))
+            for xs in self.sets:
+                xs.append(torch.zeros(m, w.k, dtype=self.xtorch, device=self.device))
             self.y.append(torch.empty(m, w.n, dtype=self.ytorch, device=self.device))
         self.ws_bytes = max(Q.qvla_linear_workspace_bytes(layer, m) for layer in self.layers)
         self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=self.device)
@@ -55,13 +59,21 @@ class LinearStack:
         for layer, t in zip(self.layers, tables):
             Q.qvla_set_step_scales(layer, np.asarray(t, dtype=np.float32))
 
-    def set_input(self, i: int, x) -> None:
-        self.x[i].copy_(torch.as_tensor(x).to(self.xtorch))
+    @property
+    def x(self):
+        """The inputs of the first set."""
+        return self.sets[0]
+
+    def inputs(self, step: int):
+        return self.sets[step] if len(self.sets) > 1 and step >= 0 else self.sets[0]
+
+    def set_input(self, i: int, x, input_set: int = 0) -> None:
+        self.sets[input_set][i].copy_(torch.as_tensor(x).to(self.xtorch))
 
     def run(self, step: int = -1, stream=None) -> None:
         """One pass over every layer; step -1 quantises per token, step t >= 0 with the tables."""
         stream = torch.cuda.current_stream() if stream is None else stream
-        for layer, x, y in zip(self.layers, self.x, self.y):
+        for layer, x, y in zip(self.layers, self.inputs(step), self.y):
             Q.qvla_w4a4_linear(layer, x, self.m, step, y, self.ws, self.ws_bytes, stream)
 
     def capture(self, step: int = -1) -> torch.cuda.CUDAGraph:
