@@ -85,6 +85,12 @@ def barrier(world):
         dist.barrier()
 
 
+def job_value(world: int, ops_per_step: float, steps: int, ms: float) -> float:
+    """Whole-job TOPS: every rank runs `steps` steps of its own replica (weak scaling); `ms` is
+    the slowest rank's time."""
+    return world * ops_per_step * steps / (ms * 1e-3) / 1e12
+
+
 def max_over_ranks(world, value: float, device) -> float:
     if world == 1:
         return value
@@ -255,7 +261,7 @@ def run_ours(args):
     gemm_gu_ms = sum(e[1].elapsed_time(e[2]) for e in evs.values()) / ne
     rqh_ms = sum(e[2].elapsed_time(e[3]) for e in evs.values()) / ne
     gemm_dn_ms = sum(e[3].elapsed_time(e[4]) for e in evs.values()) / ne
-    value = world * OPS_STEP * K / (ms * 1e-3) / 1e12
+    value = job_value(world, OPS_STEP, K, ms)
 
     # ---- end to end through the public API with host buffers ----
     x_host = mlp.x.pin_memory()
@@ -276,7 +282,7 @@ def run_ours(args):
     barrier(world)
     Q.qvla_check_device(stream)
     ms2 = max_over_ranks(world, e0.elapsed_time(e1), dev)
-    e2e = world * OPS_STEP * K2 / (ms2 * 1e-3) / 1e12
+    e2e = job_value(world, OPS_STEP, K2, ms2)
 
     peak_tflops, peak_gbs, peak_src = peaks()
     stacks = None if args.no_stacks else run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src)

@@ -374,14 +374,17 @@ cudaError_t launch_t(const RotQuantArgs& a) {
   const size_t smem = (kLogB > ((kEpt == 128) ? 7 : 6)) ? static_cast<size_t>(tpb) * kEpt * sizeof(float) : 0;
   auto kern = rotate_quant_kernel<T, kLogB, kEpt, kStep>;
   if (smem > 48 * 1024) {
-    // raise the shared-memory limit once per device (bit d of the mask)
+    // raise the kernel's limit once per device to the most any K asks of it (one kernel serves
+    // several K, so several sizes: at most 256 threads x 128 float32 = 128 KB)
+    constexpr int kMaxSmem = 128 * 1024;
+    if (smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
     static std::atomic<unsigned long long> raised{0};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     const unsigned long long bit = 1ull << (dev & 63);
     if (!(raised.load() & bit)) {
-      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
       if (e != cudaSuccess) return e;
       raised.fetch_or(bit);
     }
