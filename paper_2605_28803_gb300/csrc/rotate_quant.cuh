@@ -64,16 +64,12 @@ struct Loader<float> {
   }
 };
 
-__device__ __forceinline__ void bfly2(float2& a, float2& c) {  // (a, c) -> (a + c, a - c), two lanes at once
-  float2 s, d;
-  asm("{\n.reg .b64 ra, rc, rs, rd;\n"
-      "mov.b64 ra, {%4, %5};\nmov.b64 rc, {%6, %7};\n"
-      "add.rn.f32x2 rs, ra, rc;\nsub.rn.f32x2 rd, ra, rc;\n"
-      "mov.b64 {%0, %1}, rs;\nmov.b64 {%2, %3}, rd;\n}\n"
-      : "=f"(s.x), "=f"(s.y), "=f"(d.x), "=f"(d.y)
-      : "f"(a.x), "f"(a.y), "f"(c.x), "f"(c.y));
+// (a, c) -> (a + c, a - c), two lanes at once; a - c as one rounding of c * (-1) + a, the same
+// value a subtraction gives.
+__device__ __forceinline__ void bfly2(float2& a, float2& c) {
+  const float2 s = __fadd2_rn(a, c);
+  c = __ffma2_rn(c, make_float2(-1.0f, -1.0f), a);
   a = s;
-  c = d;
 }
 
 // Butterflies on element-index bits [lo, hi) of v (kN float2 = 2 kN elements; bit 0 is the
@@ -113,15 +109,11 @@ static __device__ __noinline__ float exact_code(float y, float c, float delta, f
   return q + kMagic;
 }
 
-// 8 codes (as kMagic + q floats) -> one packed word, code 2j in the low nibble of byte j.
-__device__ __forceinline__ uint32_t pack8(const float (&u)[8]) {
-  uint32_t b[4];
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const uint32_t lo = __float_as_uint(u[2 * j]), hi = __float_as_uint(u[2 * j + 1]) << 4;
-    b[j] = (lo & 0x0Fu) | (hi & 0xF0u);
-  }
-  return __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
+// The low bytes of four words, in order, as one word.  A code held as the float kMagic + q has
+// q's two's-complement low byte as the low byte of its bits.
+__device__ __forceinline__ uint32_t low_bytes(float a, float b, float c, float d) {
+  return __byte_perm(__byte_perm(__float_as_uint(a), __float_as_uint(b), 0x0040),
+                     __byte_perm(__float_as_uint(c), __float_as_uint(d), 0x0040), 0x5410);
 }
 
 // Sum of the 8 two's-complement codes of a packed word, plus 64 (each code offset by 8).
@@ -253,27 +245,36 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
   // codes in register order, 8 per word (register element r = 8 g + i)
   uint32_t pk[kEpt / 8];
   uint32_t sum_acc = 0;
+  const float2 cr2 = make_float2(cr, cr);
+  const float2 magic2 = make_float2(kMagic, kMagic), nmagic2 = make_float2(-kMagic, -kMagic);
+  const float2 neg2 = make_float2(-1.0f, -1.0f);
 #pragma unroll
   for (int g = 0; g < kEpt / 8; ++g) {
-    float u[8];
-    bool tie = false;
+    // elements 8 g + 2 i (.x) and 8 g + 2 i + 1 (.y), as kMagic + code, two at a time
+    float2 u[4];
+    float dev = 0.0f;  // the largest distance |t - round(t)| of the 8
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int idx = 8 * g + i;
-      const float y = (idx & 1) ? v[idx >> 1].y : v[idx >> 1].x;
-      float t = y * cr;
-      if constexpr (kStep) t = fminf(fmaxf(t, -7.0f), 7.0f);
-      u[i] = t + kMagic;
-      tie |= fabsf(t - (u[i] - kMagic)) >= kTieBand;
+    for (int i = 0; i < 4; ++i) {
+      float2 t = __fmul2_rn(v[4 * g + i], cr2);
+      if constexpr (kStep) {
+        t.x = fminf(fmaxf(t.x, -7.0f), 7.0f);
+        t.y = fminf(fmaxf(t.y, -7.0f), 7.0f);
+      }
+      u[i] = __fadd2_rn(t, magic2);
+      const float2 d = __ffma2_rn(__fadd2_rn(u[i], nmagic2), neg2, t);  // t - round(t)
+      dev = fmaxf(dev, fmaxf(fabsf(d.x), fabsf(d.y)));
     }
-    if (tie || tiny_scale) {  // rare: decide these values exactly
+    if (dev >= kTieBand || tiny_scale) {  // rare: decide these values exactly
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int idx = 8 * g + i;
-        u[i] = exact_code((idx & 1) ? v[idx >> 1].y : v[idx >> 1].x, inv_sqrt_b, delta, cr);
+      for (int i = 0; i < 4; ++i) {
+        u[i].x = exact_code(v[4 * g + i].x, inv_sqrt_b, delta, cr);
+        u[i].y = exact_code(v[4 * g + i].y, inv_sqrt_b, delta, cr);
       }
     }
-    pk[g] = pack8(u);
+    // byte j of the packed word: code 8 g + 2 j (low nibble) and 8 g + 2 j + 1 (high nibble)
+    const uint32_t even = low_bytes(u[0].x, u[1].x, u[2].x, u[3].x);
+    const uint32_t odd = low_bytes(u[0].y, u[1].y, u[2].y, u[3].y);
+    pk[g] = (even & 0x0F0F0F0Fu) | ((odd << 4) & 0xF0F0F0F0u);
     sum_acc = sum8_offset(pk[g], sum_acc);
   }
 
