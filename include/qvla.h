@@ -82,6 +82,25 @@ qvla_status qvla_pack_weights_host(const void* W, qvla_dtype wdt, int N, int K,
                                    const double* rot, int rot_block, const int32_t* perm,
                                    int had_block, uint8_t* wq, float* wscale, int32_t* wsum);
 
+/* The data-dependent factors of the composite rotation, chosen offline from the weights alone
+ * (Sec. 4.1, Eq. 4 and the permutation P that follows it).  Host only.
+ *   perm: input channels sorted by descending energy sum_n W[n,k]^2 (ties: lower channel
+ *         first) and dealt across the K / block blocks in zigzag order -- forwards in even
+ *         rounds, backwards in odd ones -- each block taking its channels in dealing order;
+ *         column j of W.P is column perm[j] of W.
+ *   rot:  for each block b of block channels of W.P, U_b = the block x block left singular
+ *         vectors of the paper's row partition W_b = (W.P)[:, block b]^T, columns by
+ *         descending singular value, each column's largest-magnitude entry positive; stored
+ *         as qvla_pack_weights_host takes it (rot_block = block).
+ * Pass both to qvla_pack_weights_host (with any Hadamard block that is a multiple of block) and
+ * apply x . P . BlockDiag(U_b) to the activations upstream (reading: the library's online
+ * rotation is the Hadamard factor).
+ *   W     host [N][K] of dtype wdt.   block  divides K, 1 <= block <= 512.
+ *   perm  host out int32 [K].          rot    host out float64 [K/block][block][block].
+ * ------------------------------------------------------------------------------------------ */
+qvla_status qvla_block_svd_rotation(const void* W, qvla_dtype wdt, int N, int K, int block, int32_t* perm,
+                                    double* rot);
+
 /* Upload already-packed weights as a layer (synchronous; allocates device memory the layer
  * owns).  wq host [N][K/2], wscale host [N], bias host [N] float32 or NULL.  xdt is the
  * activation dtype the layer accepts (F16, BF16 or F32); ydt the output dtype (F16 or BF16).

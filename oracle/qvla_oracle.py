@@ -9,6 +9,9 @@ share no code (no kernels, headers, tables, helpers, pre- or post-processing).
 What is computed, in the paper's order (Sec. 4):
   * Sec. 4.1, Eq. 3-5: the composite rotation X' = X P R_hat, W' = P^T R_hat^T W with
     R_hat = BlockDiag(U_b H_c).  Written out as dense float64 products.
+  * Sec. 4.1 (Eq. 4 and the permutation after it): the offline choice of P (channels sorted
+    by weight energy, dealt across blocks in zigzag order) and of U_b (the left singular
+    vectors of each block's row partition, from numpy's SVD).
   * Sec. 4.2, Eq. 5: Delta_Z = max|Z| / q_max, q_max = 2^(k-1) - 1 = 7 at k = 4.
   * Sec. 4.2, Eq. 6 (first display): Q_Z = clamp(round(Z / Delta_Z), -q_max, q_max).
   * Sec. 4.2: weight scales per output channel, backbone activation scales per token,
@@ -33,6 +36,11 @@ Readings of the paper that this file fixes (each is also listed in the design no
   R6  Packed int4: byte j of a row holds code 2j in its low nibble and code 2j+1 in
       its high nibble, each as a 4-bit two's-complement integer.
   R7  The down-projection glue of the gated MLP is gelu_tanh(gate) * up.
+  R14 The zigzag deals the energy-sorted channels (ties: lower index first) forwards in even
+      rounds and backwards in odd ones; Eq. 5's W' = P^T R_hat^T W is read as the fold that
+      keeps X W unchanged, R_hat^T P^T W.
+  R15 U_b's columns are ordered by descending singular value, each signed so that its
+      largest-magnitude entry is positive (the SVD fixes them only up to sign).
 
 Functions with no pin in the paper (the paper prints no worked numeric example) are
 pinned by closed forms, invariants, library special cases and brute force in
@@ -142,6 +150,47 @@ def fold_weights(w: np.ndarray, had_block: int, perm=None, rot=None, rot_block=N
     wr = apply_permutation(w, perm)
     wr = apply_block_rotation(wr, rot, rot_block)
     return block_hadamard_rotate(wr, had_block)
+
+
+def zigzag_permutation(w: np.ndarray, block: int) -> np.ndarray:
+    """The channel permutation P of Sec. 4.1 (after Eq. 4): input channels sorted by descending
+    weight energy sum_n W[n, j]^2 (ties by channel index), dealt across the K/block blocks in
+    zigzag order -- round r visits the blocks forwards for even r, backwards for odd r -- each
+    block taking its channels in the order dealt.  Returns perm (int64 [K]): column j of X P is
+    column perm[j] of X, i.e. block b holds channels perm[b block : (b + 1) block]."""
+    w = np.asarray(w, dtype=np.float64)
+    k = w.shape[1]
+    if k % block:
+        raise ValueError(f"K={k} is not a multiple of the block {block}")
+    nb = k // block
+    energy = (w * w).sum(axis=0)
+    order = np.argsort(-energy, kind="stable")
+    perm = np.empty(k, dtype=np.int64)
+    for i, j in enumerate(order):
+        r, pos = divmod(i, nb)
+        b = pos if r % 2 == 0 else nb - 1 - pos
+        perm[b * block + r] = j
+    return perm
+
+
+def block_svd_rotation(w: np.ndarray, block: int, perm=None) -> np.ndarray:
+    """The SVD factors U_b of Eq. 4 for the weights stored [C_out, C_in]: after the permutation,
+    block b of the input channels is W_b = (W P)[:, b]^T (block x C_out, the paper's row
+    partition) and U_b its block x block left singular vectors, columns ordered by descending
+    singular value (reading R2 of U_SVD(W_b^T)).  Each column's sign makes its largest-magnitude
+    entry positive (the first, on a tie).  Returns rot [K/block, block, block] float64, to be
+    used as x . BlockDiag(U_b)."""
+    wp = apply_permutation(np.asarray(w, dtype=np.float64), perm)
+    k = wp.shape[1]
+    nb = k // block
+    rot = np.empty((nb, block, block), dtype=np.float64)
+    for b in range(nb):
+        wb = wp[:, b * block:(b + 1) * block].T
+        u, _, _ = np.linalg.svd(wb, full_matrices=True)
+        idx = np.argmax(np.abs(u), axis=0)
+        u = u * np.where(u[idx, np.arange(block)] < 0, -1.0, 1.0)[None, :]
+        rot[b] = u
+    return rot
 
 
 def upstream_activation_transform(x: np.ndarray, perm=None, rot=None, rot_block=None) -> np.ndarray:

@@ -152,6 +152,19 @@ qvla_status qvla_pack_weights_host(const void* W, qvla_dtype wdt, int N, int K, 
   return QVLA_OK;
 }
 
+qvla_status qvla_block_svd_rotation(const void* W, qvla_dtype wdt, int N, int K, int block, int32_t* perm,
+                                    double* rot) {
+  g_last_error.clear();
+  if (!W || !perm || !rot) return fail(QVLA_ERR_INVALID_ARG, "W, perm and rot must not be NULL");
+  if (wdt != QVLA_F16 && wdt != QVLA_BF16 && wdt != QVLA_F32) return fail(QVLA_ERR_INVALID_ARG, "bad weight dtype %d", wdt);
+  if (N <= 0 || K <= 0) return fail(QVLA_ERR_INVALID_ARG, "N=%d and K=%d must be positive", N, K);
+  if (block < 1 || block > 512 || K % block != 0)
+    return fail(QVLA_ERR_INVALID_ARG, "block=%d must be in [1, 512] and divide K=%d", block, K);
+  qvla::zigzag_permutation_host(W, static_cast<int>(wdt), N, K, block, perm);
+  qvla::block_svd_rotation_host(W, static_cast<int>(wdt), N, K, block, perm, rot);
+  return QVLA_OK;
+}
+
 static qvla_status upload_layer(int N, int K, int had_block, qvla_dtype xdt, qvla_dtype ydt, int gated,
                                 const uint8_t* wq, const float* wscale, const float* bias, qvla_layer** out) {
   if (xdt != QVLA_F16 && xdt != QVLA_BF16 && xdt != QVLA_F32) return fail(QVLA_ERR_INVALID_ARG, "bad activation dtype %d", xdt);

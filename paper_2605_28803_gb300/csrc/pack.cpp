@@ -3,6 +3,10 @@
 // to float32, then Delta_W[n] = max |W'_n| / 7 (float32) and int4 codes
 // clamp(round(W'/Delta_W), -7, 7) rounded half to even on the exact quotient, nibble-packed.
 // The Hadamard factor is applied with an in-place radix-2 fast transform.
+//
+// Also the offline choice of P and U_b (Sec. 4.1, after Eq. 4): the zigzag channel permutation
+// by weight energy, and per block of input channels the left singular vectors of the block's
+// row partition, found as the eigenvectors of its Gram matrix by cyclic Jacobi rotations.
 #include "pack.h"
 
 #include <algorithm>
@@ -138,6 +142,123 @@ void pack_weights_host_impl(const void* W, int wdt, int N, int K, const double* 
       const int n = next.fetch_add(1);
       if (n >= N) break;
       pack_row(W, wdt, K, n, rot, rot_block, perm, had_block, a, b, f, wq, wscale, wsum);
+    }
+  };
+  std::vector<std::thread> pool;
+  for (unsigned i = 1; i < nt; ++i) pool.emplace_back(worker);
+  worker();
+  for (auto& t : pool) t.join();
+}
+
+namespace {
+
+// Eigen-decomposition of a symmetric c x c matrix a (row-major, destroyed) by cyclic Jacobi
+// rotations: on return the eigenvalues are on a's diagonal and v's column j is the unit
+// eigenvector of eigenvalue a[j][j].  Each rotation zeroes one off-diagonal pair exactly in
+// exact arithmetic; sweeps repeat until the off-diagonal mass is negligible.
+void jacobi_eigen(std::vector<double>& a, std::vector<double>& v, int c) {
+  v.assign(static_cast<size_t>(c) * c, 0.0);
+  for (int i = 0; i < c; ++i) v[static_cast<size_t>(i) * c + i] = 1.0;
+  auto A = [&](int i, int j) -> double& { return a[static_cast<size_t>(i) * c + j]; };
+  auto V = [&](int i, int j) -> double& { return v[static_cast<size_t>(i) * c + j]; };
+  double total = 0.0;
+  for (int i = 0; i < c; ++i)
+    for (int j = 0; j < c; ++j) total += A(i, j) * A(i, j);
+  for (int sweep = 0; sweep < 100; ++sweep) {
+    double off = 0.0;
+    for (int p = 0; p < c; ++p)
+      for (int q = p + 1; q < c; ++q) off += A(p, q) * A(p, q);
+    if (off <= 1e-32 * total) break;
+    for (int p = 0; p < c - 1; ++p)
+      for (int q = p + 1; q < c; ++q) {
+        const double apq = A(p, q);
+        if (apq == 0.0) continue;
+        // the rotation angle that zeroes A(p, q): t = tan(phi), the smaller root
+        const double theta = (A(q, q) - A(p, p)) / (2.0 * apq);
+        const double t = (theta >= 0.0 ? 1.0 : -1.0) / (std::fabs(theta) + std::sqrt(theta * theta + 1.0));
+        const double cs = 1.0 / std::sqrt(t * t + 1.0), sn = t * cs;
+        for (int k = 0; k < c; ++k) {  // columns p and q
+          const double akp = A(k, p), akq = A(k, q);
+          A(k, p) = cs * akp - sn * akq;
+          A(k, q) = sn * akp + cs * akq;
+        }
+        for (int k = 0; k < c; ++k) {  // rows p and q
+          const double apk = A(p, k), aqk = A(q, k);
+          A(p, k) = cs * apk - sn * aqk;
+          A(q, k) = sn * apk + cs * aqk;
+        }
+        for (int k = 0; k < c; ++k) {
+          const double vkp = V(k, p), vkq = V(k, q);
+          V(k, p) = cs * vkp - sn * vkq;
+          V(k, q) = sn * vkp + cs * vkq;
+        }
+      }
+  }
+}
+
+}  // namespace
+
+void zigzag_permutation_host(const void* W, int wdt, int N, int K, int block, int32_t* perm) {
+  std::vector<double> energy(K, 0.0);
+  for (int n = 0; n < N; ++n)
+    for (int k = 0; k < K; ++k) {
+      const double w = load_elem(W, wdt, static_cast<size_t>(n) * K + k);
+      energy[k] += w * w;
+    }
+  std::vector<int> order(K);
+  for (int k = 0; k < K; ++k) order[k] = k;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return energy[a] > energy[b]; });
+  const int nb = K / block;
+  for (int i = 0; i < K; ++i) {
+    const int r = i / nb, pos = i % nb;
+    const int b = (r % 2 == 0) ? pos : nb - 1 - pos;
+    perm[b * block + r] = order[i];
+  }
+}
+
+void block_svd_rotation_host(const void* W, int wdt, int N, int K, int block, const int32_t* perm, double* rot) {
+  const int nb = K / block;
+  unsigned nt = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
+  nt = std::min<unsigned>(nt, static_cast<unsigned>(std::max(1, nb)));
+  std::atomic<int> next{0};
+  auto worker = [&]() {
+    std::vector<double> wb(static_cast<size_t>(N) * block), g(static_cast<size_t>(block) * block), v;
+    std::vector<int> idx(block);
+    for (;;) {
+      const int b = next.fetch_add(1);
+      if (b >= nb) break;
+      // the block's input channels (after P) for every output row
+      for (int n = 0; n < N; ++n)
+        for (int i = 0; i < block; ++i) {
+          const int k = b * block + i;
+          wb[static_cast<size_t>(n) * block + i] = load_elem(W, wdt, static_cast<size_t>(n) * K + (perm ? perm[k] : k));
+        }
+      // Gram matrix of the paper's row partition W_b (block x N): G = W_b W_b^T
+      std::fill(g.begin(), g.end(), 0.0);
+      for (int n = 0; n < N; ++n) {
+        const double* row = wb.data() + static_cast<size_t>(n) * block;
+        for (int i = 0; i < block; ++i) {
+          const double ri = row[i];
+          for (int j = i; j < block; ++j) g[static_cast<size_t>(i) * block + j] += ri * row[j];
+        }
+      }
+      for (int i = 0; i < block; ++i)
+        for (int j = 0; j < i; ++j) g[static_cast<size_t>(i) * block + j] = g[static_cast<size_t>(j) * block + i];
+      jacobi_eigen(g, v, block);
+      // columns by descending eigenvalue (= sigma^2), each with its largest entry positive
+      for (int i = 0; i < block; ++i) idx[i] = i;
+      std::stable_sort(idx.begin(), idx.end(), [&](int a, int c) {
+        return g[static_cast<size_t>(a) * block + a] > g[static_cast<size_t>(c) * block + c];
+      });
+      double* u = rot + static_cast<size_t>(b) * block * block;
+      for (int j = 0; j < block; ++j) {
+        const int src = idx[j];
+        int arg = 0;
+        for (int i = 1; i < block; ++i)
+          if (std::fabs(v[static_cast<size_t>(i) * block + src]) > std::fabs(v[static_cast<size_t>(arg) * block + src])) arg = i;
+        const double sgn = v[static_cast<size_t>(arg) * block + src] < 0.0 ? -1.0 : 1.0;
+        for (int i = 0; i < block; ++i) u[static_cast<size_t>(i) * block + j] = sgn * v[static_cast<size_t>(i) * block + src];
+      }
     }
   };
   std::vector<std::thread> pool;

@@ -9,6 +9,10 @@ namespace qvla {
 void pack_weights_host_impl(const void* W, int wdt, int N, int K, const double* rot, int rot_block,
                             const int32_t* perm, int had_block, uint8_t* wq, float* wscale, int32_t* wsum);
 
+// The zigzag channel permutation by weight energy and the block SVD factors (Sec. 4.1).
+void zigzag_permutation_host(const void* W, int wdt, int N, int K, int block, int32_t* perm);
+void block_svd_rotation_host(const void* W, int wdt, int N, int K, int block, const int32_t* perm, double* rot);
+
 // wsum[n] = sum of the int4 codes of packed row n.
 void code_sums_host(const uint8_t* wq, int N, int K, int32_t* wsum);
 

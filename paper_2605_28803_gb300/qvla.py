@@ -27,6 +27,7 @@ SIGNATURES = {
     "qvla_last_error": (ctypes.c_char_p, []),
     "qvla_abi_version": (_I, []),
     "qvla_pack_weights_host": (_I, [_P, _I, _I, _I, _P, _I, _P, _I, _P, _P, _P]),
+    "qvla_block_svd_rotation": (_I, [_P, _I, _I, _I, _I, _P, _P]),
     "qvla_layer_create": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, ctypes.POINTER(_P)]),
     "qvla_layer_create_gated": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, ctypes.POINTER(_P)]),
     "qvla_pack_weights": (_I, [_P, _I, _I, _I, _P, _I, _P, _I, _P, _I, _I, ctypes.POINTER(_P)]),
@@ -99,6 +100,16 @@ def qvla_pack_weights_host(W: np.ndarray, wdt: int, N: int, K: int, rot=None, ro
     """Host-only fold + quantise + pack into caller-provided numpy buffers."""
     _check(_lib.qvla_pack_weights_host(_ptr(W), wdt, N, K, _ptr(rot), rot_block, _ptr(perm), had_block,
                                        _ptr(wq), _ptr(wscale), _ptr(wsum)))
+
+
+def qvla_block_svd_rotation(W: np.ndarray, wdt: int, N: int, K: int, block: int):
+    """The zigzag permutation and block SVD factors chosen from the weights; returns
+    (perm int32 [K], rot float64 [K/block, block, block])."""
+    perm = np.empty(max(K, 1), dtype=np.int32)
+    ok = block > 0 and K > 0 and K % block == 0
+    rot = np.empty((K // block, block, block) if ok else (1,), dtype=np.float64)  # the library rejects bad shapes
+    _check(_lib.qvla_block_svd_rotation(_ptr(np.ascontiguousarray(W)), wdt, N, K, block, _ptr(perm), _ptr(rot)))
+    return perm, rot
 
 
 class Layer:

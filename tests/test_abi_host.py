@@ -113,3 +113,36 @@ def test_host_pack_dense_svd_factor_config1():
     wq, ws, _ = _host_pack(case.w, Q.F32, case.had_block, rot=np.ascontiguousarray(case.rot), rot_block=case.rot_block)
     oq, osc, _ = O.pack_weights(case.w.astype(np.float64), case.had_block, rot=case.rot, rot_block=case.rot_block)
     assert np.array_equal(ws, osc) and np.array_equal(wq, oq)
+
+
+def test_block_svd_rotation_matches_oracle():
+    """The library's offline factors (Sec. 4.1): the zigzag permutation equals the oracle's
+    exactly; the block SVD factors agree to 1e-9 (Jacobi on the Gram matrix against LAPACK's
+    SVD, same column order and sign rule)."""
+    rng = np.random.default_rng(31)
+    for N, K, block in [(96, 512, 64), (40, 256, 32), (256, 128, 128)]:
+        w = (W.gaussian_weights(rng, N, K, 0.02) * rng.uniform(0.2, 4.0, K)[None, :]).astype(np.float32)
+        perm, rot = Q.qvla_block_svd_rotation(w, Q.F32, N, K, block)
+        operm = O.zigzag_permutation(w, block)
+        orot = O.block_svd_rotation(w, block, operm)
+        assert np.array_equal(perm, operm)
+        assert np.abs(rot - orot).max() < 1e-9, (N, K, block)
+
+
+def test_pack_with_library_svd_factors_matches_oracle():
+    rng = np.random.default_rng(32)
+    N, K, block = 64, 512, 64
+    w = (W.gaussian_weights(rng, N, K, 0.02) * rng.uniform(0.2, 4.0, K)[None, :]).astype(np.float32)
+    perm, rot = Q.qvla_block_svd_rotation(w, Q.F32, N, K, block)
+    wq, ws, _ = _host_pack(w, Q.F32, 256, rot=rot, rot_block=block, perm=perm)
+    oq, osc, oc = O.pack_weights(w.astype(np.float64), 256, perm=perm, rot=rot, rot_block=block)
+    assert np.array_equal(ws, osc)
+    assert np.array_equal(O.unpack_int4(wq), oc)
+
+
+def test_block_svd_rotation_rejects_bad_block():
+    w = np.zeros((4, 96), np.float32)
+    for block in (0, 7, 1024):
+        with pytest.raises(Q.QvlaError) as e:
+            Q.qvla_block_svd_rotation(w, Q.F32, 4, 96, block)
+        assert e.value.status == 1

@@ -167,3 +167,28 @@ def test_linear_halves_equal_whole_call():
     Q.qvla_check_device(G.stream())
     assert np.array_equal(y.double().cpu().numpy(), whole)
     layer.close()
+
+
+def test_linear_with_block_svd_and_zigzag_rotation():
+    """The full composite rotation of Sec. 4.1 (Eq. 4-5): P and U_b chosen from the weights by
+    the library (zigzag permutation, block SVD with block 64, the paper's setting), folded with
+    Hadamard 512; the activations get x . P . BlockDiag(U_b) upstream (float64, rounded once to
+    fp16) and the online path runs per token.  Both sides use the same factors."""
+    rng = np.random.default_rng(41)
+    M, N, K, block, had = 96, 384, 1024, 64, 512
+    w = (W.gaussian_weights(rng, N, K, 0.02) * rng.uniform(0.2, 4.0, K)[None, :]).astype(np.float32)
+    x = W.gaussian_with_outliers(rng, M, K, 5, 20.0)
+    perm, rot = Q.qvla_block_svd_rotation(w, Q.F32, N, K, block)
+    wq = np.zeros((N, K // 2), np.uint8)
+    ws = np.zeros(N, np.float32)
+    Q.qvla_pack_weights_host(w, Q.F32, N, K, rot=rot, rot_block=block, perm=perm, had_block=had, wq=wq, wscale=ws)
+    layer = G.make_layer(wq, ws, had, "f16", "f16")
+    x_up = W.as_dtype(O.upstream_activation_transform(x, perm, rot, block), "f16")
+    got = G.linear(layer, x_up, ydt="f16")
+    _, oscale, codes = O.pack_weights(w.astype(np.float64), had, perm=perm, rot=rot, rot_block=block)
+    ref = O.w4a4_linear(x_up.double().numpy(), codes, oscale, had, out_fmt="f16")
+    G.assert_output_close(got, ref["y"], "f16")
+    # the quantised layer still approximates the float one (the rotation is orthogonal)
+    exact = x.astype(np.float64) @ w.astype(np.float64).T
+    assert O.relative_output_error(got, exact) < 0.35
+    layer.close()

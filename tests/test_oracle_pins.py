@@ -98,6 +98,74 @@ def check_rotation_invariance(o):
         assert not np.allclose(xr, x)
 
 
+def check_zigzag_golden(o):
+    g = read_golden("zigzag_worked.txt")
+    w = np.array([[float(v) for v in g["w"]]])
+    perm = o.zigzag_permutation(w, int(g["block"][0]))
+    assert perm.tolist() == [int(v) for v in g["perm"]]
+    energy = (w * w).sum(axis=0)
+    assert [energy[perm[:4]].sum(), energy[perm[4:]].sum()] == [float(v) for v in g["block_energy"]]
+
+
+def check_zigzag_rule(o):
+    """The i-th channel of the energy order lands in block i mod 2nb, or 2nb - 1 - (i mod 2nb)
+    past the turn (the zigzag written as one index formula), in dealing order; the result is a
+    permutation and spreads energy more evenly than contiguous blocks of the sorted list."""
+    rng = np.random.default_rng(21)
+    for k, block in [(256, 64), (64, 8), (96, 32)]:
+        w = rng.standard_normal((40, k)) * rng.uniform(0.1, 5.0, k)[None, :]
+        perm = o.zigzag_permutation(w, block)
+        assert sorted(perm.tolist()) == list(range(k))
+        nb = k // block
+        energy = (w * w).sum(axis=0)
+        order = sorted(range(k), key=lambda j: (-energy[j], j))
+        expect = [[] for _ in range(nb)]
+        for i, j in enumerate(order):
+            t = i % (2 * nb)
+            expect[t if t < nb else 2 * nb - 1 - t].append(j)
+        assert perm.tolist() == [j for blk in expect for j in blk]
+        be = energy[perm].reshape(nb, block).sum(axis=1)
+        bc = np.sort(energy)[::-1].reshape(nb, block).sum(axis=1)
+        assert be.max() - be.min() < bc.max() - bc.min()
+
+
+def check_block_svd_golden(o):
+    g = read_golden("svd_worked.txt")
+    w = np.array([[float(v) for v in g["w_row0"]], [float(v) for v in g["w_row1"]]])
+    u = np.array([[float(v) for v in g["u_times_sqrt10_row0"]], [float(v) for v in g["u_times_sqrt10_row1"]]])
+    rot = o.block_svd_rotation(w, 2)
+    assert np.allclose(rot[0], u / math.sqrt(10.0), rtol=0, atol=1e-14)
+    rows = rot[0].T @ w.T
+    assert np.allclose((rows * rows).sum(axis=1), [float(v) for v in g["sigma_squared"]], rtol=1e-13)
+
+
+def check_block_svd_properties(o):
+    """Each U_b is orthogonal; the rows of U_b^T W_b carry energies sigma_i^2 in descending
+    order (Sec. 4.1: the rotated block's row energy is its singular spectrum), with sigma from
+    scipy's svdvals; the largest entry of every column is positive; and the composite fold
+    with P and these U_b still preserves X W^T."""
+    rng = np.random.default_rng(22)
+    k, n, block = 128, 48, 32
+    w = rng.standard_normal((n, k)) * rng.uniform(0.2, 3.0, k)[None, :]
+    perm = o.zigzag_permutation(w, block)
+    rot = o.block_svd_rotation(w, block, perm)
+    wp = w[:, perm]
+    for b in range(k // block):
+        u = rot[b]
+        assert np.allclose(u.T @ u, np.eye(block), atol=1e-13)
+        wb = wp[:, b * block:(b + 1) * block].T
+        rows = u.T @ wb
+        sig = scipy.linalg.svdvals(wb)
+        assert np.allclose((rows * rows).sum(axis=1), sig ** 2, rtol=1e-10)
+        idx = np.argmax(np.abs(u), axis=0)
+        assert np.all(u[idx, np.arange(block)] > 0)
+    x = rng.standard_normal((5, k))
+    xr = o.block_hadamard_rotate(o.upstream_activation_transform(x, perm, rot, block), 64)
+    wr = o.fold_weights(w, 64, perm, rot, block)
+    ref = x @ w.T
+    assert np.allclose(xr @ wr.T, ref, rtol=1e-11, atol=1e-11 * np.abs(ref).max())
+
+
 def check_quantizer_golden(o):
     g = read_golden("quantizer_worked.txt")
     z = np.array([float(v) for v in g["z"]], dtype=np.float32)
@@ -291,6 +359,7 @@ PINS = {f.__name__: f for f in [
     check_pack_golden_and_roundtrip, check_int_gemm_bruteforce, check_round_to_format,
     check_linear_golden, check_dequant_special_cases, check_step_lookup, check_calibration,
     check_weight_roundtrip, check_end_to_end_band,
+    check_zigzag_golden, check_zigzag_rule, check_block_svd_golden, check_block_svd_properties,
 ]}
 
 
@@ -315,6 +384,7 @@ _real_quantize = O.quantize
 _real_int_gemm = O.int_gemm
 _real_dequant = O.dequant_output
 _real_apply_block_rotation = O.apply_block_rotation
+_real_block_svd = O.block_svd_rotation
 _real_round = O.round_to_format
 
 
@@ -402,6 +472,25 @@ def _mut_round_truncate(x, fmt):
     return out
 
 
+def _mut_zigzag_round_robin(w, block):
+    w = np.asarray(w, np.float64)
+    k = w.shape[1]
+    nb = k // block
+    order = np.argsort(-(w * w).sum(axis=0), kind="stable")
+    perm = np.empty(k, dtype=np.int64)
+    for i, j in enumerate(order):
+        perm[(i % nb) * block + i // nb] = j
+    return perm
+
+
+def _mut_svd_ascending(w, block, perm=None):
+    return _real_block_svd(w, block, perm)[:, :, ::-1].copy()
+
+
+def _mut_svd_transposed(w, block, perm=None):
+    return np.transpose(_real_block_svd(w, block, perm), (0, 2, 1)).copy()
+
+
 MUTANTS = {
     "hadamard_wrong_order": ("sylvester_hadamard", _mut_hadamard_order),
     "rotate_unnormalised": ("block_hadamard_rotate", _mut_rotate_unnormalised),
@@ -418,6 +507,9 @@ MUTANTS = {
     "dequant_bias_twice": ("dequant_output", _mut_dequant_bias_twice),
     "step_lookup_off_by_one": ("step_scale_lookup", _mut_lookup_off_by_one),
     "round_truncates": ("round_to_format", _mut_round_truncate),
+    "zigzag_without_turns": ("zigzag_permutation", _mut_zigzag_round_robin),
+    "svd_columns_ascending": ("block_svd_rotation", _mut_svd_ascending),
+    "svd_factor_transposed_in_pack": ("block_svd_rotation", _mut_svd_transposed),
 }
 
 
