@@ -203,20 +203,25 @@ def upstream_activation_transform(x: np.ndarray, perm=None, rot=None, rot_block=
 # Sec. 4.2 -- symmetric uniform quantiser
 # --------------------------------------------------------------------------------------
 
-def absmax_scale(z: np.ndarray, axis=None) -> np.ndarray:
+def qmax_of(bits: int) -> int:
+    """q_max = 2^(k-1) - 1 for k-bit symmetric codes (Sec. 4.2, Eq. 5): 7 at k = 4, 127 at k = 8."""
+    return 2 ** (bits - 1) - 1
+
+
+def absmax_scale(z: np.ndarray, axis=None, qmax: int = QMAX) -> np.ndarray:
     """Delta_Z = max|Z| / q_max (Sec. 4.2, Eq. 5), in float32 as the stored scale.
 
     z must already be float32 (the values the quantiser sees).  The maximum of float32
-    magnitudes is exact; the division by 7 is one IEEE float32 division.
+    magnitudes is exact; the division by q_max is one IEEE float32 division.
     """
     z = np.asarray(z)
     if z.dtype != np.float32:
         raise TypeError("absmax_scale expects float32 input")
     m = np.max(np.abs(z), axis=axis)
-    return (np.asarray(m, dtype=np.float32) / np.float32(QMAX)).astype(np.float32)
+    return (np.asarray(m, dtype=np.float32) / np.float32(qmax)).astype(np.float32)
 
 
-def quantize(z: np.ndarray, delta: np.ndarray) -> np.ndarray:
+def quantize(z: np.ndarray, delta: np.ndarray, qmax: int = QMAX) -> np.ndarray:
     """Q_Z = clamp(round(Z / Delta), -q_max, q_max) (Sec. 4.2, Eq. 6), int8 codes.
 
     z and delta are float32 (delta broadcasts against z).  Reading R4: round() is
@@ -236,7 +241,7 @@ def quantize(z: np.ndarray, delta: np.ndarray) -> np.ndarray:
         r = np.rint(z64 / d64)
     r = np.where(d64 == 0.0, 0.0, r)
     r = np.where(np.isnan(r), 0.0, r)
-    return np.clip(r, -QMAX, QMAX).astype(np.int8)
+    return np.clip(r, -qmax, qmax).astype(np.int8)
 
 
 def dequantize(q: np.ndarray, delta: np.ndarray) -> np.ndarray:
@@ -304,11 +309,11 @@ def rotate_activations(x: np.ndarray, had_block: int) -> np.ndarray:
     return block_hadamard_rotate(np.asarray(x, dtype=np.float64), had_block).astype(np.float32)
 
 
-def quantize_activations_per_token(y: np.ndarray):
+def quantize_activations_per_token(y: np.ndarray, qmax: int = QMAX):
     """Backbone activations: one scale per token (Sec. 4.2), Eq. 5-6 along each row.
     y: float32 [M, K] rotated activations.  Returns (codes int8 [M, K], scales f32 [M])."""
-    scale = absmax_scale(y, axis=1)
-    return quantize(y, scale[:, None]), scale
+    scale = absmax_scale(y, axis=1, qmax=qmax)
+    return quantize(y, scale[:, None], qmax), scale
 
 
 def step_scale_lookup(table, t: int) -> np.float32:
@@ -320,11 +325,11 @@ def step_scale_lookup(table, t: int) -> np.float32:
     return table[t]
 
 
-def quantize_activations_per_step(y: np.ndarray, table, t: int):
+def quantize_activations_per_step(y: np.ndarray, table, t: int, qmax: int = QMAX):
     """DiT activations: the step-t scale replaces Delta_Z in Eq. 6 (Sec. 4.2)."""
     d = step_scale_lookup(table, t)
     scale = np.full(y.shape[0], d, dtype=np.float32)
-    return quantize(y, scale[:, None]), scale
+    return quantize(y, scale[:, None], qmax), scale
 
 
 def robust_peak(y: np.ndarray, estimator: str = "absmax") -> np.float32:
@@ -408,18 +413,21 @@ def dequant_output(acc: np.ndarray, dx: np.ndarray, dw: np.ndarray, bias=None, o
 
 
 def w4a4_linear(x: np.ndarray, w_codes: np.ndarray, w_scale: np.ndarray, had_block: int,
-                bias=None, table=None, step: int | None = None, out_fmt: str = "f16"):
+                bias=None, table=None, step: int | None = None, out_fmt: str = "f16", act_bits: int = 4):
     """The online quantized linear of Sec. 4: rotate (Eq. 5), quantise per token or with
     the step-t table scale (Eq. 5-6), integer GEMM and dequantisation (Eq. 7).
 
     x: activations [M, K] already in the P.U basis (reading R2), as fp16/bf16/fp32 values.
+    act_bits: 4 (W4A4) or 8 (W4A8, the paper's deployed precision: the same recipe with
+    k = 8, q_max = 127, for the activations only).
     Returns a dict with the rotated activations, codes, scales, int accumulator and y.
     """
+    qmax = qmax_of(act_bits)
     y32 = rotate_activations(x, had_block)
     if step is None:
-        qx, dx = quantize_activations_per_token(y32)
+        qx, dx = quantize_activations_per_token(y32, qmax)
     else:
-        qx, dx = quantize_activations_per_step(y32, table, step)
+        qx, dx = quantize_activations_per_step(y32, table, step, qmax)
     acc = int_gemm(qx, w_codes)
     out = dequant_output(acc, dx, w_scale, bias, out_fmt)
     return {"y_rot": y32, "qx": qx, "dx": dx, "acc": acc, "y": out}

@@ -166,6 +166,50 @@ def check_block_svd_properties(o):
     assert np.allclose(xr @ wr.T, ref, rtol=1e-11, atol=1e-11 * np.abs(ref).max())
 
 
+def check_quantizer_8bit_bruteforce(o):
+    """k = 8 (q_max = 127, Eq. 5): Delta = max / 127 and each code is the nearest candidate in
+    [-127, 127], ties to even, by exhaustive search in exact float64 arithmetic."""
+    rng = np.random.default_rng(23)
+    z = (rng.standard_normal(3000) * 5).astype(np.float32)
+    z[:4] = [0.5, -1.5, 2.5, 3.5]
+    d = o.absmax_scale(z, qmax=127)
+    assert d == np.float32(np.float32(np.max(np.abs(z))) / np.float32(127))
+    codes = o.quantize(z, np.float32(1.0), 127)
+    assert codes[:4].tolist() == [0, -2, 2, 4]
+    q = o.quantize(z, d, 127)
+    cand = np.arange(-127, 128, dtype=np.float64)
+    t = z.astype(np.float64) / np.float64(d)
+    dist = np.abs(t[:, None] - cand[None, :])
+    best = dist.min(axis=1)
+    for i in range(len(z)):
+        c = cand[dist[i] == best[i]]
+        expect = c[0] if len(c) == 1 else c[np.argmin(np.abs(c) % 2)]
+        assert q[i] == expect
+    assert q.min() >= -127 and q.max() <= 127 and np.count_nonzero(np.abs(q) == 127) >= 1
+
+
+def check_w4a8_linear(o):
+    """The W4A8 linear is the same recipe with 8-bit activation codes: its integer product is
+    the exhaustive sum of int8 x int4 codes, and on outlier-heavy data it approximates the
+    float product better than W4A4."""
+    rng = np.random.default_rng(24)
+    m, n, k, had = 6, 10, 64, 64
+    x = rng.standard_normal((m, k))
+    x[:, 3] *= 20
+    w = rng.standard_normal((n, k)) * 0.05
+    _, ws, wc = o.pack_weights(w, had)
+    r8 = o.w4a4_linear(x, wc, ws, had, out_fmt="f32", act_bits=8)
+    r4 = o.w4a4_linear(x, wc, ws, had, out_fmt="f32", act_bits=4)
+    assert np.abs(r8["qx"]).max() == 127 and np.abs(r4["qx"]).max() == 7
+    acc = np.zeros((m, n), dtype=np.int64)
+    for i in range(m):
+        for j in range(n):
+            acc[i, j] = sum(int(r8["qx"][i, t]) * int(wc[j, t]) for t in range(k))
+    assert np.array_equal(r8["acc"], acc)
+    ref = x @ w.T
+    assert o.relative_output_error(r8["y"], ref) < o.relative_output_error(r4["y"], ref)
+
+
 def check_quantizer_golden(o):
     g = read_golden("quantizer_worked.txt")
     z = np.array([float(v) for v in g["z"]], dtype=np.float32)
@@ -360,6 +404,7 @@ PINS = {f.__name__: f for f in [
     check_linear_golden, check_dequant_special_cases, check_step_lookup, check_calibration,
     check_weight_roundtrip, check_end_to_end_band,
     check_zigzag_golden, check_zigzag_rule, check_block_svd_golden, check_block_svd_properties,
+    check_quantizer_8bit_bruteforce, check_w4a8_linear,
 ]}
 
 
@@ -472,6 +517,10 @@ def _mut_round_truncate(x, fmt):
     return out
 
 
+def _mut_quantize_ignores_qmax(z, d, qmax=7):
+    return _real_quantize(z, d, 7)
+
+
 def _mut_zigzag_round_robin(w, block):
     w = np.asarray(w, np.float64)
     k = w.shape[1]
@@ -508,6 +557,7 @@ MUTANTS = {
     "step_lookup_off_by_one": ("step_scale_lookup", _mut_lookup_off_by_one),
     "round_truncates": ("round_to_format", _mut_round_truncate),
     "zigzag_without_turns": ("zigzag_permutation", _mut_zigzag_round_robin),
+    "quantize_8bit_clamps_at_7": ("quantize", _mut_quantize_ignores_qmax),
     "svd_columns_ascending": ("block_svd_rotation", _mut_svd_ascending),
     "svd_factor_transposed_in_pack": ("block_svd_rotation", _mut_svd_transposed),
 }
