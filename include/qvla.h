@@ -233,6 +233,47 @@ qvla_status qvla_linear_gemm(const qvla_layer* layer, const void* workspace, siz
 qvla_status qvla_w4a4_linear_noalloc(const qvla_layer* layer, const void* x, int M, int step, void* y,
                                      void* stream);
 
+/* ------------------------------------------------------------------------------------------
+ * W4A8 variant (the appendix on the real-quantization kernel, "Real-Quantization Kernel
+ * Implementation", Table 5): the same int4 weights of the layer against 8-bit activation codes,
+ * with the same scales and epilogue.  Per token (step == -1) the scale is max_k |y_k| / 127;
+ * per step it is the table entry as given (a table calibrated for 8-bit codes holds
+ * absmax / 127); codes are clamp(round(y / xscale[m]), -127, 127), round half to even on the
+ * exact quotient of the float32 operands.  With had_block == 1 no rotation runs at all, the
+ * appendix's configuration (rotations folded into the weights offline).
+ *
+ * The accumulator stays exact for K <= 4096 (255 x 15 x K < 2^24 units of the tensor cores'
+ * float32 accumulator); layers with a longer K return QVLA_ERR_UNSUPPORTED.
+ * ------------------------------------------------------------------------------------------ */
+
+/* Rotate + quantise to 8-bit codes: as qvla_rotate_quantize_rows with q_max = 127.
+ *   xq device out [M][K] int8 codes, natural k order, 16-byte aligned.
+ *   xscale device out [M] float32; xsum device out [M] int32 or NULL (sum of row m's codes). */
+qvla_status qvla_rotate_quantize_rows_a8(const void* x, qvla_dtype xdt, int M, int K, int had_block,
+                                         const float* step_scale, int8_t* xq, float* xscale,
+                                         int32_t* xsum, void* stream);
+
+/* Bytes of device workspace qvla_w4a8_linear and qvla_gemm_w4a8 need for M rows (a multiple of
+ * 256): the codes as two tensor-core operand planes (M x 2K bytes), the scales and the sums. */
+size_t qvla_w4a8_workspace_bytes(const qvla_layer* layer, int M);
+
+/* The whole W4A8 linear: rotate + quantise x to 8-bit codes (step as in qvla_rotate_quantize),
+ * then the integer GEMM and the epilogue of qvla_gemm_w4a4 on them.  x device [M][K], y device
+ * out [M][N] (H for a gated layer); workspace as for qvla_w4a4_linear but of
+ * qvla_w4a8_workspace_bytes(layer, M) bytes. */
+qvla_status qvla_w4a8_linear(const qvla_layer* layer, const void* x, int M, int step, void* y,
+                             void* workspace, size_t workspace_bytes, void* stream);
+
+/* Integer GEMM + epilogue on 8-bit codes quantised elsewhere (e.g. by
+ * qvla_rotate_quantize_rows_a8):  acc[m,n] = sum_k xq[m,k] * wq[n,k] (exact),
+ * y[m,n] = ydt(fma((float)acc[m,n], xscale[m] * Delta_W[n], bias[n])).
+ *   xq device [M][K] int8 (16-byte aligned), xscale device [M];
+ *   y device out, acc device out [M][N] int32 or NULL (test hook), as in qvla_gemm_w4a4;
+ *   workspace of qvla_w4a8_workspace_bytes(layer, M) bytes, 256-byte aligned (the operand
+ *   planes and the code sums are built there first). */
+qvla_status qvla_gemm_w4a8(const qvla_layer* layer, const int8_t* xq, const float* xscale, int M, void* y,
+                           int32_t* acc, void* workspace, size_t workspace_bytes, void* stream);
+
 /* Synchronise `stream`, then report (and clear) the device-side error word: QVLA_OK, or
  * QVLA_ERR_TIMEOUT if a kernel gave up waiting since the last check. */
 qvla_status qvla_check_device(void* stream);

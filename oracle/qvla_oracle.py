@@ -364,14 +364,15 @@ def int_gemm(qx: np.ndarray, qw: np.ndarray) -> np.ndarray:
     """acc[m, n] = sum_k Q_X'[m, k] Q_W'[n, k]: the integer product of Eq. 7, int64.
 
     Evaluated with a float64 matrix product: every product is an integer of magnitude
-    <= 64 and every partial sum an integer of magnitude <= 64 K < 2^53, all exactly
-    representable, so the result is the exact integer whatever the summation order.
+    <= 128 x 8 = 1024 (8-bit activation codes against int4 weights; <= 64 for int4 x int4) and
+    every partial sum an integer of magnitude <= 1024 K < 2^53, all exactly representable, so
+    the result is the exact integer whatever the summation order.
     """
     qx = np.asarray(qx)
     qw = np.asarray(qw)
     if qx.shape[-1] != qw.shape[-1]:
         raise ValueError("reduction lengths differ")
-    if qx.shape[-1] * 64 >= 2 ** 53:
+    if qx.shape[-1] * 1024 >= 2 ** 53:
         raise ValueError("K too large for an exact float64 product")
     return (qx.astype(np.float64) @ qw.astype(np.float64).T).astype(np.int64)
 

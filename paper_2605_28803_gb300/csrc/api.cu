@@ -22,6 +22,7 @@ struct qvla_layer {
   uint8_t* wq = nullptr;      // device, tiled: [groups][K/128][128 rows][64 B] (see upload_layer)
   float* wscale = nullptr;    // device [N]
   float* wcorr = nullptr;     // device [N]: 8 * (sum of the codes of row n), the GEMM's offset correction
+  float* wcorr8 = nullptr;    // device [N]: 128 * (sum of the codes of row n), the same for 8-bit activations
   float* bias = nullptr;      // device [N] (zeros when the layer was given none)
   float* table = nullptr;     // device [table_cap]
   int T = 0, table_cap = 0;
@@ -92,7 +93,7 @@ qvla_status check_rows(int M) {
 }
 
 qvla_status launch_rq(const void* x, int xdt, int M, int K, int had_block, int mode, const float* step_scale,
-                      uint8_t* xq, float* xscale, int32_t* xsum, float* absmax, void* stream, int out_bytes = 0) {
+                      uint8_t* xq, float* xscale, int32_t* xsum, float* absmax, void* stream, int out_mode = 0) {
   qvla::RotQuantArgs a;
   a.x = x;
   a.xdt = xdt;
@@ -106,7 +107,7 @@ qvla_status launch_rq(const void* x, int xdt, int M, int K, int had_block, int m
   a.xscale = xscale;
   a.xsum = xsum;
   a.absmax = absmax;
-  a.out_bytes = out_bytes;
+  a.out_mode = out_mode;
   a.stream = static_cast<cudaStream_t>(stream);
   QVLA_CUDA(qvla::launch_rotate_quant(a), "rotate_quantize launch");
   return QVLA_OK;
@@ -173,8 +174,11 @@ static qvla_status upload_layer(int N, int K, int had_block, qvla_dtype xdt, qvl
     if (!(wscale[n] >= 0.0f) || std::isinf(wscale[n])) return fail(QVLA_ERR_INVALID_ARG, "wscale[%d] is not a finite non-negative float", n);
   std::vector<int32_t> wsum(N);
   qvla::code_sums_host(wq, N, K, wsum.data());
-  std::vector<float> wcorr(N), zero_bias;
-  for (int n = 0; n < N; ++n) wcorr[n] = 8.0f * static_cast<float>(wsum[n]);  // exact: |8 wsum| <= 2^20
+  std::vector<float> wcorr(N), wcorr8(N), zero_bias;
+  for (int n = 0; n < N; ++n) {
+    wcorr[n] = 8.0f * static_cast<float>(wsum[n]);      // exact: |8 wsum| <= 2^20
+    wcorr8[n] = 128.0f * static_cast<float>(wsum[n]);   // exact: |128 wsum| <= 2^24
+  }
   if (!bias) {
     zero_bias.assign(N, 0.0f);
     bias = zero_bias.data();
@@ -210,10 +214,12 @@ static qvla_status upload_layer(int N, int K, int had_block, qvla_dtype xdt, qvl
   cudaError_t e = cudaMalloc(&L->wq, wbytes);
   if (e == cudaSuccess) e = cudaMalloc(&L->wscale, N * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&L->wcorr, N * sizeof(float));
+  if (e == cudaSuccess) e = cudaMalloc(&L->wcorr8, N * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&L->bias, N * sizeof(float));
   if (e == cudaSuccess) e = cudaMemcpy(L->wq, tiled.data(), wbytes, cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(L->wscale, wscale, N * sizeof(float), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(L->wcorr, wcorr.data(), N * sizeof(float), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(L->wcorr8, wcorr8.data(), N * sizeof(float), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(L->bias, bias, N * sizeof(float), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     qvla_layer_destroy(L);
@@ -287,6 +293,7 @@ qvla_status qvla_layer_destroy(qvla_layer* L) {
   cudaFree(L->wq);
   cudaFree(L->wscale);
   cudaFree(L->wcorr);
+  cudaFree(L->wcorr8);
   cudaFree(L->bias);
   cudaFree(L->table);
   delete L;
@@ -358,6 +365,20 @@ qvla_status qvla_rotated_absmax(const void* x, qvla_dtype xdt, int M, int K, int
   return launch_rq(x, xdt, M, K, had_block, 2, nullptr, nullptr, nullptr, nullptr, absmax, stream);
 }
 
+qvla_status qvla_rotate_quantize_rows_a8(const void* x, qvla_dtype xdt, int M, int K, int had_block,
+                                         const float* step_scale, int8_t* xq, float* xscale, int32_t* xsum,
+                                         void* stream) {
+  g_last_error.clear();
+  if (qvla_status s = check_rows(M)) return s;
+  if (qvla_status s = check_shape(16, K, had_block)) return s;
+  if (xdt != QVLA_F16 && xdt != QVLA_BF16 && xdt != QVLA_F32) return fail(QVLA_ERR_INVALID_ARG, "bad activation dtype %d", xdt);
+  if (M == 0) return QVLA_OK;
+  if (!x || !xq || !xscale) return fail(QVLA_ERR_INVALID_ARG, "x, xq and xscale must not be NULL");
+  if (!aligned16(x) || !aligned16(xq)) return fail(QVLA_ERR_INVALID_ARG, "x and xq must be 16-byte aligned");
+  return launch_rq(x, xdt, M, K, had_block, step_scale ? 1 : 0, step_scale, reinterpret_cast<uint8_t*>(xq), xscale,
+                   xsum, nullptr, stream, 2);
+}
+
 }  // extern "C"
 
 namespace {
@@ -370,7 +391,7 @@ qvla_status launch_gemm(const qvla_layer* L, const uint8_t* xq, int x_bytes, con
   a.xsum = xsum;
   a.wq = L->wq;
   a.wscale = L->wscale;
-  a.wcorr = L->wcorr;
+  a.wcorr = x_bytes == 2 ? L->wcorr8 : L->wcorr;
   a.bias = L->bias;
   a.y = y;
   a.ydt = L->ydt;
@@ -470,6 +491,80 @@ qvla_status qvla_w4a4_linear(const qvla_layer* L, const void* x, int M, int step
   if (qvla_status s = launch_rq(x, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr, stream, 1))
     return s;
   return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream);
+}
+
+}  // extern "C"
+
+// ---- W4A8: 8-bit activation codes against the same int4 weights ----
+namespace {
+constexpr int kMaxKA8 = 4096;  // the FP32 accumulator is exact while 255 x 15 x K < 2^24
+
+qvla_status check_a8(const qvla_layer* L) {
+  if (L->K > kMaxKA8)
+    return fail(QVLA_ERR_UNSUPPORTED, "K=%d: 8-bit activations need K <= %d (exact accumulation)", L->K, kMaxKA8);
+  return QVLA_OK;
+}
+
+struct A8Workspace {
+  uint8_t* planes;   // [M][2K] operand planes
+  float* xscale;     // [M]
+  int32_t* xsum;     // [M]
+};
+
+qvla_status carve_a8(const qvla_layer* L, int M, void* workspace, size_t workspace_bytes, A8Workspace* w) {
+  if (!workspace) return fail(QVLA_ERR_INVALID_ARG, "workspace must not be NULL");
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u) return fail(QVLA_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  const size_t need = qvla_w4a8_workspace_bytes(L, M);
+  if (workspace_bytes < need)
+    return fail(QVLA_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed", workspace_bytes, need);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  w->planes = ws;
+  w->xscale = reinterpret_cast<float*>(ws + round256(static_cast<size_t>(M) * 2 * L->K));
+  w->xsum = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(w->xscale) + round256(static_cast<size_t>(M) * 4));
+  return QVLA_OK;
+}
+}  // namespace
+
+extern "C" {
+
+size_t qvla_w4a8_workspace_bytes(const qvla_layer* L, int M) {
+  if (!L || M <= 0) return 0;
+  return round256(static_cast<size_t>(M) * 2 * L->K) + round256(static_cast<size_t>(M) * 4) * 2;
+}
+
+qvla_status qvla_w4a8_linear(const qvla_layer* L, const void* x, int M, int step, void* y, void* workspace,
+                             size_t workspace_bytes, void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_a8(L)) return s;
+  if (qvla_status s = check_rows(M)) return s;
+  const float* ss = nullptr;
+  if (qvla_status s = resolve_step(L, step, &ss)) return s;
+  if (M == 0) return QVLA_OK;
+  if (!x || !y) return fail(QVLA_ERR_INVALID_ARG, "x and y must not be NULL");
+  if (!aligned16(x) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "x and y must be 16-byte aligned");
+  A8Workspace w;
+  if (qvla_status s = carve_a8(L, M, workspace, workspace_bytes, &w)) return s;
+  if (qvla_status s = launch_rq(x, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.planes, w.xscale, w.xsum, nullptr,
+                                stream, 3))
+    return s;
+  return launch_gemm(L, w.planes, 2, w.xscale, w.xsum, M, y, nullptr, stream);
+}
+
+qvla_status qvla_gemm_w4a8(const qvla_layer* L, const int8_t* xq, const float* xscale, int M, void* y, int32_t* acc,
+                           void* workspace, size_t workspace_bytes, void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_a8(L)) return s;
+  if (qvla_status s = check_rows(M)) return s;
+  if (M == 0) return QVLA_OK;
+  if (!xq || !xscale || !y) return fail(QVLA_ERR_INVALID_ARG, "xq, xscale and y must not be NULL");
+  if (!aligned16(xq) || !aligned16(y) || !aligned16(acc))
+    return fail(QVLA_ERR_INVALID_ARG, "xq, y and acc must be 16-byte aligned");
+  A8Workspace w;
+  if (qvla_status s = carve_a8(L, M, workspace, workspace_bytes, &w)) return s;
+  QVLA_CUDA(qvla::launch_a8_planes(xq, M, L->K, w.planes, w.xsum, static_cast<cudaStream_t>(stream)), "a8 planes launch");
+  return launch_gemm(L, w.planes, 2, xscale, w.xsum, M, y, acc, stream);
 }
 
 }  // extern "C"

@@ -61,10 +61,14 @@ constexpr uint32_t kEpiBarrier = 1;  // named barrier of the epilogue warps
 
 // kStageA / kStageB: whether operand A / B of the MMA arrives packed (staged, then expanded by
 // the converters); otherwise it arrives as operand bytes straight from a swizzled TMA load.
-template <int kBN, bool kStageA = true, bool kStageB = true>
+// kPlanes: operand-byte planes per k-block of the activations (2 for 8-bit codes: the high and
+// the low nibbles, each one 128-byte tile against the same weight tile).
+template <int kBN, bool kStageA = true, bool kStageB = true, int kPlanes = 1>
 struct Cfg {
-  static constexpr int kTileA = kBM * kBK;    // bytes of E4M3
-  static constexpr int kTileB = kBN * kBK;
+  static constexpr int kTileA1 = kBM * kBK;   // bytes of E4M3 of one plane
+  static constexpr int kTileB1 = kBN * kBK;
+  static constexpr int kTileA = kTileA1 * (kStageA ? 1 : kPlanes);
+  static constexpr int kTileB = kTileB1 * (kStageB ? 1 : kPlanes);
   static constexpr int kStage = kTileA + kTileB;             // expanded k-block
   static constexpr int kRawA = kStageA ? kBM * kBK / 2 : 0;  // packed k-block (64-byte rows)
   static constexpr int kRawB = kStageB ? kBN * kBK / 2 : 0;
@@ -94,6 +98,7 @@ struct Params {
   int M, N;      // N = weight rows of the layer (2H for a gated layer)
   int ldy;       // row length of y (N, or H for a gated layer)
   int splits;    // weight-major orientation: CTAs of a cluster splitting K (1 = no split)
+  float kconst;  // the zero-point constant of the accumulator: 64 K (int4 codes), 1024 K (int8)
 };
 
 __device__ __forceinline__ void epi_sync() {
@@ -170,12 +175,12 @@ __device__ __forceinline__ void store_row32(OutT* dst, const uint32_t (&pk)[16],
 // Epilogue parameters of 4 consecutive weight rows n .. n + 3 and one token m (split-K reduction);
 // indices past the end are clamped so the loads can be issued unconditionally.
 struct SplitParams {
-  float cm, xs;       // 64 K + 8 xsum[m], xscale[m]
+  float cm, xs;       // kconst + 8 xsum[m], xscale[m]
   float4 wc, ws, bs;  // wcorr, wscale, bias of rows n .. n + 3
   __device__ __forceinline__ void load(const Params& p, int n, int m) {
     n = min(n, p.N - 4);
     m = min(m, p.M - 1);
-    cm = 64.0f * static_cast<float>(p.K) + 8.0f * static_cast<float>(__ldg(p.xsum + m));
+    cm = p.kconst + 8.0f * static_cast<float>(__ldg(p.xsum + m));
     xs = __ldg(p.xscale + m);
     wc = __ldg(reinterpret_cast<const float4*>(p.wcorr + n));
     ws = __ldg(reinterpret_cast<const float4*>(p.wscale + n));
@@ -183,15 +188,19 @@ struct SplitParams {
   }
 };
 
-// kXBytes: the activations arrive as operand bytes ([rows][K], written by the rotate-quantise
-// kernel) and are TMA-loaded with the 128-byte swizzle straight into the MMA operand tile; only
-// the weights are staged and expanded.  Otherwise both operands are packed int4.
-template <int kBN, bool kSwap, bool kGated, bool kXBytes, typename OutT>
+// kX: how the activations arrive.  0: packed int4, staged and expanded like the weights.
+// 1: operand bytes ([rows][K], written by the rotate-quantise kernel), TMA-loaded with the
+// 128-byte swizzle straight into the MMA operand tile; only the weights are staged and
+// expanded.  2: the two operand planes of 8-bit codes ([rows][2K]: per k-block the high then
+// the low nibbles), both loaded per k-block and multiplied with the same expanded weight tile.
+template <int kBN, bool kSwap, bool kGated, int kX, typename OutT>
 __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_constant__ CUtensorMap tmap_a,
                                                                  const __grid_constant__ CUtensorMap tmap_b, Params p) {
+  constexpr bool kXBytes = kX >= 1;
+  constexpr int kPlanes = kX == 2 ? 2 : 1;
   constexpr bool kStageA = !(kXBytes && !kSwap);  // operand A is the activations unless swapped
   constexpr bool kStageB = !(kXBytes && kSwap);
-  using C = Cfg<kBN, kStageA, kStageB>;
+  using C = Cfg<kBN, kStageA, kStageB, kPlanes>;
   static_assert(kSwap || kBN % 128 == 0, "a weight tile is whole 128-row chunks");
   extern __shared__ uint8_t dyn_smem[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~uintptr_t(1023));
@@ -309,10 +318,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
             const uint32_t e = smem_u32(smem + s * C::kStage);
             if constexpr (!kSwap) {
               mbar_arrive_expect_tx(fb, C::kTileA);
-              tma_load_2d(e, &tmap_a, kb * kBK, ta * kBM, fb);
+#pragma unroll
+              for (int pl = 0; pl < kPlanes; ++pl)
+                tma_load_2d(e + pl * C::kTileA1, &tmap_a, (kb * kPlanes + pl) * kBK, ta * kBM, fb);
             } else {
               mbar_arrive_expect_tx(fb, C::kTileB);
-              tma_load_2d(e + C::kTileA, &tmap_b, kb * kBK, tb * kBN, fb);
+#pragma unroll
+              for (int pl = 0; pl < kPlanes; ++pl)
+                tma_load_2d(e + C::kTileA + pl * C::kTileB1, &tmap_b, (kb * kPlanes + pl) * kBK, tb * kBN, fb);
             }
           }
         }
@@ -386,9 +399,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
           const uint32_t sa = smem_u32(smem + s * C::kStage);
           const uint32_t sb = sa + C::kTileA;
 #pragma unroll
-          for (int kk = 0; kk < kBK / 32; ++kk) {
-            mma_e4m3(d, smem_desc_sw128(sa + kk * 32), smem_desc_sw128(sb + kk * 32), kIdesc,
-                     (kb != kb0 || kk != 0) ? 1u : 0u);
+          for (int pl = 0; pl < kPlanes; ++pl) {
+            // plane pl of the activations against the same weight tile
+            const uint32_t pa = sa + (kStageA ? 0 : pl * C::kTileA1);
+            const uint32_t pb = sb + (kStageB ? 0 : pl * C::kTileB1);
+#pragma unroll
+            for (int kk = 0; kk < kBK / 32; ++kk) {
+              mma_e4m3(d, smem_desc_sw128(pa + kk * 32), smem_desc_sw128(pb + kk * 32), kIdesc,
+                       (kb != kb0 || pl != 0 || kk != 0) ? 1u : 0u);
+            }
           }
           mma_commit(smem_u32(&bar_empty[s]));
         }
@@ -404,7 +423,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     // ------------------------------------------------------------------ epilogue
     const int et = threadIdx.x;  // 0..127 = TMEM lane
     int tile_iter = 0;
-    const float k64 = 64.0f * static_cast<float>(p.K);
+    const float k64 = p.kconst;
     griddep_wait();  // xscale / xsum come from the previous kernel, and y may still be read by it
     for (int tile = QVLA_UNIT0; tile < ntiles; tile += QVLA_NUNITS, ++tile_iter) {
       const int ta = tile % tiles_a, tb = tile / tiles_a;
@@ -734,11 +753,13 @@ int max_active_clusters(const void* kern, const cudaLaunchConfig_t& cfg) {
   return n;
 }
 
-template <int kBN, bool kSwap, bool kGated, bool kXBytes, typename OutT>
+template <int kBN, bool kSwap, bool kGated, int kX, typename OutT>
 cudaError_t launch_cfg(const GemmArgs& a) {
+  constexpr bool kXBytes = kX >= 1;
+  constexpr int kPlanes = kX == 2 ? 2 : 1;
   constexpr bool kStageA = !(kXBytes && !kSwap);
   constexpr bool kStageB = !(kXBytes && kSwap);
-  using C = Cfg<kBN, kStageA, kStageB>;
+  using C = Cfg<kBN, kStageA, kStageB, kPlanes>;
   Params p;
   if (kSwap) {
     p.a = a.wq;
@@ -752,6 +773,7 @@ cudaError_t launch_cfg(const GemmArgs& a) {
     p.rows_b = a.N;
   }
   p.K = a.K;
+  p.kconst = (kX == 2 ? 1024.0f : 64.0f) * static_cast<float>(a.K);
   p.xscale = a.xscale;
   p.xsum = a.xsum;
   p.wscale = a.wscale;
@@ -764,7 +786,7 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   p.ldy = a.gated ? a.N / 2 : a.N;
   const int tiles = ((p.rows_a + kBM - 1) / kBM) * ((p.rows_b + kBN - 1) / kBN);
   if (tiles == 0) return cudaSuccess;
-  auto kern = gemm_w4a4_kernel<kBN, kSwap, kGated, kXBytes, OutT>;
+  auto kern = gemm_w4a4_kernel<kBN, kSwap, kGated, kX, OutT>;
   cudaError_t e = prepare_kernel(reinterpret_cast<const void*>(kern), C::kSmem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -800,9 +822,11 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   // a tensor map for the activations only (the weights arrive as contiguous chunks)
   CUtensorMap ta = {}, tb = {};
   if constexpr (kSwap) {
-    e = kStageB ? make_tmap(&tb, p.b, p.rows_b, p.K / 2, kBN) : make_tmap_bytes(&tb, p.b, p.rows_b, p.K, kBN);
+    e = kStageB ? make_tmap(&tb, p.b, p.rows_b, p.K / 2, kBN)
+                : make_tmap_bytes(&tb, p.b, p.rows_b, kPlanes * p.K, kBN);
   } else {
-    e = kStageA ? make_tmap(&ta, p.a, p.rows_a, p.K / 2, kBM) : make_tmap_bytes(&ta, p.a, p.rows_a, p.K, kBM);
+    e = kStageA ? make_tmap(&ta, p.a, p.rows_a, p.K / 2, kBM)
+                : make_tmap_bytes(&ta, p.a, p.rows_a, kPlanes * p.K, kBM);
   }
   if (e != cudaSuccess) return e;
   e = cudaLaunchKernelEx(&cfg, kern, ta, tb, p);
@@ -810,31 +834,32 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   return cudaGetLastError();
 }
 
-template <bool kXBytes, typename OutT>
+template <int kX, typename OutT>
 cudaError_t launch_out(const GemmArgs& a) {
-  if (a.gated) return launch_cfg<256, false, true, kXBytes, OutT>(a);  // gate/up pairs share a 256-row tile
+  if (a.gated) return launch_cfg<256, false, true, kX, OutT>(a);  // gate/up pairs share a 256-row tile
   if (a.M > 128) {
     // tile width by estimated time: waves of persistent CTAs x tile width (a narrower tile
     // wins when the wide one leaves SMs idle, e.g. few output channels and a long K)
     const long tm = (a.M + kBM - 1) / kBM;
     const long w256 = (tm * ((a.N + 255) / 256) + a.num_sms - 1) / a.num_sms;
     const long w128 = (tm * ((a.N + 127) / 128) + a.num_sms - 1) / a.num_sms;
-    if (w128 * 128 < w256 * 256) return launch_cfg<128, false, false, kXBytes, OutT>(a);
-    return launch_cfg<256, false, false, kXBytes, OutT>(a);
+    if (w128 * 128 < w256 * 256) return launch_cfg<128, false, false, kX, OutT>(a);
+    return launch_cfg<256, false, false, kX, OutT>(a);
   }
   const int mpad = (a.M + 15) / 16 * 16;
-  if (mpad <= 16) return launch_cfg<16, true, false, kXBytes, OutT>(a);
-  if (mpad <= 32) return launch_cfg<32, true, false, kXBytes, OutT>(a);
-  if (mpad <= 64) return launch_cfg<64, true, false, kXBytes, OutT>(a);
-  return launch_cfg<128, true, false, kXBytes, OutT>(a);
+  if (mpad <= 16) return launch_cfg<16, true, false, kX, OutT>(a);
+  if (mpad <= 32) return launch_cfg<32, true, false, kX, OutT>(a);
+  if (mpad <= 64) return launch_cfg<64, true, false, kX, OutT>(a);
+  return launch_cfg<128, true, false, kX, OutT>(a);
 }
 
 }  // namespace
 
 cudaError_t launch_gemm_w4a4(const GemmArgs& a) {
   if (a.M == 0) return cudaSuccess;
-  if (a.x_bytes) return a.ydt == 0 ? launch_out<true, __half>(a) : launch_out<true, __nv_bfloat16>(a);
-  return a.ydt == 0 ? launch_out<false, __half>(a) : launch_out<false, __nv_bfloat16>(a);
+  if (a.x_bytes == 2) return a.ydt == 0 ? launch_out<2, __half>(a) : launch_out<2, __nv_bfloat16>(a);
+  if (a.x_bytes == 1) return a.ydt == 0 ? launch_out<1, __half>(a) : launch_out<1, __nv_bfloat16>(a);
+  return a.ydt == 0 ? launch_out<0, __half>(a) : launch_out<0, __nv_bfloat16>(a);
 }
 
 cudaError_t read_and_clear_error_word(unsigned int* out, cudaStream_t stream) {

@@ -17,8 +17,11 @@ struct RotQuantArgs {
   float inv_sqrt_b;        // float32(1 / sqrt(b))
   int mode;                // 0 per-token, 1 per-step (step_scale), 2 absmax only
   const float* step_scale; // device, one float (mode 1)
-  uint8_t* xq;             // device [M][K/2] packed codes, or [M][K] operand bytes (out_bytes)
-  int out_bytes;           // 1: one E4M3 operand byte per code (the GEMM's internal encoding)
+  uint8_t* xq;             // device output, by out_mode:
+  int out_mode;            // 4-bit codes: 0 packed nibbles [M][K/2]; 1 one E4M3 operand byte per
+                           //   code [M][K] (the GEMM's internal encoding);
+                           // 8-bit codes: 2 int8 rows [M][K]; 3 the GEMM's two operand planes
+                           //   [M][2K] (per 128 codes: high nibbles, then low nibbles)
   float* xscale;           // device [M]
   int32_t* xsum;           // device [M] or null
   float* absmax;           // device, one float (mode 2)
@@ -27,16 +30,23 @@ struct RotQuantArgs {
 bool rotate_quant_supported(int log_b);
 cudaError_t launch_rotate_quant(const RotQuantArgs& a);
 
+// ---- int8 codes to the W4A8 GEMM's operand planes (a8_planes.cu) ----
+// xq: device [M][K] int8 codes (16-byte aligned rows); planes: device [M][2K]; xsum: device [M]
+// or null (cleared, then the codes' row sums added).
+cudaError_t launch_a8_planes(const int8_t* xq, int M, int K, uint8_t* planes, int32_t* xsum, cudaStream_t stream);
+
 // ---- W4A4 GEMM + epilogue (gemm.cu) ----
 struct GemmArgs {
-  const uint8_t* xq;       // device [M][K/2] activation codes, or [M][K] operand bytes (x_bytes)
-  int x_bytes;             // 1: xq holds the rotate-quantise kernel's operand bytes
+  const uint8_t* xq;       // device activations, by x_bytes:
+  int x_bytes;             // 0: packed int4 codes [M][K/2]; 1: the rotate-quantise kernel's
+                           //   operand bytes of int4 codes [M][K]; 2: its two operand planes of
+                           //   int8 codes [M][2K] (the W4A8 variant, K <= 4096)
   const float* xscale;     // device [M]
   const int32_t* xsum;     // device [M]
   const uint8_t* wq;       // device weight codes, tiled: 8 KB chunks of 128 rows x 128 codes,
                            // [groups][K/128][128][64 B], groups even (rows past N are zero)
   const float* wscale;     // device [N]
-  const float* wcorr;      // device [N]: 8 * sum_k wq[n,k] as float
+  const float* wcorr;      // device [N]: 8 * sum_k wq[n,k] as float (128 * sum for x_bytes 2)
   const float* bias;       // device [N] (zeros when the layer has no bias)
   void* y;                 // device [M][N], dtype ydt
   int ydt;                 // 0 f16, 1 bf16

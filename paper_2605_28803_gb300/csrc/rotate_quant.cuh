@@ -6,9 +6,10 @@
 // runs its butterfly stages on the low log2(EPT) index bits in registers (stages of distance
 // >= 2 as packed f32x2 adds/subs), then transposes once through shared memory so that each
 // thread holds the elements that differ in the remaining bits, and runs those in registers
-// too.  The scale (per token: max |y| / 7; or the step's table entry), the int4 codes, their
-// packing and the row's code sum follow from registers.  Instantiated per input dtype in
-// rotate_quant_{f16,bf16,f32}.cu.
+// too.  The scale (per token: max |y| / q_max; or the step's table entry), the codes, their
+// packing and the row's code sum follow from registers.  Codes are int4 (q_max 7) or, for the
+// W4A8 variant, int8 (q_max 127).  Instantiated per input dtype and code width in
+// rotate_quant_{f16,bf16,f32}.cu (4-bit) and rotate_quant_a8_{f16,bf16,f32}.cu (8-bit).
 #pragma once
 
 #include <cuda_bf16.h>
@@ -18,6 +19,7 @@
 #include <atomic>
 #include <cstdint>
 
+#include "a8_codes.cuh"
 #include "griddep.cuh"
 #include "kernels.h"
 
@@ -28,6 +30,8 @@ constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23: t + kMagic rounds |t| < 2^
 // The fast path t = y * (c / delta) is within 2^-20 of the exact z / delta (|t| <= 8); a value
 // closer than this to a half-integer is decided exactly instead.
 constexpr float kTieBand = 0.5f - 7.62939453125e-6f;  // 0.5 - 2^-17
+// With 8-bit codes |t| <= 128, so the fast path is within 2^-15: a wider band, 2^-12.
+constexpr float kTieBand8 = 0.5f - 2.44140625e-4f;
 
 template <typename T>
 struct Loader;
@@ -92,20 +96,20 @@ __device__ __forceinline__ void fwht_regs(float2 (&v)[kN]) {
   }
 }
 
-// The exact decision for one value (rare: only within 2^-17 of a tie, or when 1/delta
-// overflows): round half to even of the exact quotient z / delta for z = float32(y * c), by
-// the sign of z - h delta (one FMA is exact in sign) at the half-integer h next to t, then the
-// clamp.  Returns kMagic + q.
-static __device__ __noinline__ float exact_code(float y, float c, float delta, float cr) {
+// The exact decision for one value (rare: only near a tie, or when 1/delta overflows): round
+// half to even of the exact quotient z / delta for z = float32(y * c), by the sign of
+// z - h delta (one FMA is exact in sign) at the half-integer h next to t, then the clamp to
+// [-qmax, qmax].  Returns kMagic + q.
+static __device__ __noinline__ float exact_code(float y, float c, float delta, float cr, float qmax, float band) {
   const float z = y * c;
-  if (isinf(cr)) return fminf(fmaxf(__fdiv_rn(z, delta), -7.0f), 7.0f) + kMagic;  // tiny delta
-  const float t = fminf(fmaxf(y * cr, -7.0f), 7.0f);
-  if (fabsf(t - ((t + kMagic) - kMagic)) < kTieBand) return t + kMagic;  // not near a tie
+  if (isinf(cr)) return fminf(fmaxf(__fdiv_rn(z, delta), -qmax), qmax) + kMagic;  // tiny delta
+  const float t = fminf(fmaxf(y * cr, -qmax), qmax);
+  if (fabsf(t - ((t + kMagic) - kMagic)) < band) return t + kMagic;  // not near a tie
   const float fl = floorf(t);
   const float d = fmaf(-(fl + 0.5f), delta, z);
   float q = d > 0.0f ? fl + 1.0f : fl;
   if (d == 0.0f) q = (static_cast<int>(fl) & 1) ? fl + 1.0f : fl;
-  q = fminf(fmaxf(q, -7.0f), 7.0f);
+  q = fminf(fmaxf(q, -qmax), qmax);
   return q + kMagic;
 }
 
@@ -125,13 +129,16 @@ __device__ __forceinline__ uint32_t sum8_offset(uint32_t w, uint32_t acc) {
 
 // kLogB: log2 of the Hadamard block (0 = no rotation).  kEpt: elements per thread.
 // kStep: the scale is the step table entry (else per token; per-token mode also serves the
-// calibration max when absmax_out is set).
-template <typename T, int kLogB, int kEpt, bool kStep>
+// calibration max when absmax_out is set).  kA8: 8-bit codes (q_max 127; out_mode int8 rows
+// or the GEMM's two operand planes), else 4-bit (q_max 7; packed nibbles or operand bytes).
+template <typename T, int kLogB, int kEpt, bool kStep, bool kA8>
 __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__ x, int M, int K, float inv_sqrt_b,
                                                              const float* __restrict__ step_scale,
                                                              uint8_t* __restrict__ xq, float* __restrict__ xscale,
                                                              int32_t* __restrict__ xsum, float* __restrict__ absmax_out,
-                                                             int out_bytes) {
+                                                             int out_mode) {
+  constexpr float kQ = kA8 ? 127.0f : 7.0f;
+  constexpr float kBand = kA8 ? kTieBand8 : kTieBand;
   constexpr int kP = (kEpt == 128) ? 7 : 6;  // log2(kEpt)
   static_assert((1 << kP) == kEpt, "EPT");
   constexpr int kN = kEpt / 2;                // float2 per thread
@@ -233,7 +240,7 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
       if (active && j == 0) atomicMax(reinterpret_cast<unsigned int*>(absmax_out), __float_as_uint(zmax));
       return;
     }
-    delta = __fdiv_rn(zmax, 7.0f);
+    delta = __fdiv_rn(zmax, kQ);
   }
   if (active && j == 0) xscale[m] = delta;
 
@@ -243,7 +250,9 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
   const bool tiny_scale = !zero_scale && isinf(rcp);  // 1/delta overflows: plain division
   const float cr = inv_sqrt_b * rcp;                  // y * cr ~ z / delta (0 when delta = 0: codes 0)
   // codes in register order, 8 per word (register element r = 8 g + i)
-  uint32_t pk[kEpt / 8];
+  // 4-bit: pk = packed nibbles; 8-bit: ev / od = the two's-complement code bytes of the even /
+  // odd elements of each group of 8
+  uint32_t pk[kA8 ? 1 : kEpt / 8], ev[kA8 ? kEpt / 8 : 1], od[kA8 ? kEpt / 8 : 1];
   uint32_t sum_acc = 0;
   const float2 cr2 = make_float2(cr, cr);
   const float2 magic2 = make_float2(kMagic, kMagic), nmagic2 = make_float2(-kMagic, -kMagic);
@@ -257,29 +266,37 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
     for (int i = 0; i < 4; ++i) {
       float2 t = __fmul2_rn(v[4 * g + i], cr2);
       if constexpr (kStep) {
-        t.x = fminf(fmaxf(t.x, -7.0f), 7.0f);
-        t.y = fminf(fmaxf(t.y, -7.0f), 7.0f);
+        t.x = fminf(fmaxf(t.x, -kQ), kQ);
+        t.y = fminf(fmaxf(t.y, -kQ), kQ);
       }
       u[i] = __fadd2_rn(t, magic2);
       const float2 d = __ffma2_rn(__fadd2_rn(u[i], nmagic2), neg2, t);  // t - round(t)
       dev = fmaxf(dev, fmaxf(fabsf(d.x), fabsf(d.y)));
     }
-    if (dev >= kTieBand || tiny_scale) {  // rare: decide these values exactly
+    if (dev >= kBand || tiny_scale) {  // rare: decide these values exactly
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        u[i].x = exact_code(v[4 * g + i].x, inv_sqrt_b, delta, cr);
-        u[i].y = exact_code(v[4 * g + i].y, inv_sqrt_b, delta, cr);
+        u[i].x = exact_code(v[4 * g + i].x, inv_sqrt_b, delta, cr, kQ, kBand);
+        u[i].y = exact_code(v[4 * g + i].y, inv_sqrt_b, delta, cr, kQ, kBand);
       }
     }
     // byte j of the packed word: code 8 g + 2 j (low nibble) and 8 g + 2 j + 1 (high nibble)
     const uint32_t even = low_bytes(u[0].x, u[1].x, u[2].x, u[3].x);
     const uint32_t odd = low_bytes(u[0].y, u[1].y, u[2].y, u[3].y);
-    pk[g] = (even & 0x0F0F0F0Fu) | ((odd << 4) & 0xF0F0F0F0u);
-    sum_acc = sum8_offset(pk[g], sum_acc);
+    if constexpr (kA8) {
+      ev[g] = even;
+      od[g] = odd;
+      sum_acc = __dp4a(even ^ 0x80808080u, 0x01010101u, sum_acc);  // sum of q + 128
+      sum_acc = __dp4a(odd ^ 0x80808080u, 0x01010101u, sum_acc);
+    } else {
+      pk[g] = (even & 0x0F0F0F0Fu) | ((odd << 4) & 0xF0F0F0F0u);
+      sum_acc = sum8_offset(pk[g], sum_acc);
+    }
   }
 
   // ---- store: run r holds register elements [r kRun, (r + 1) kRun), contiguous in the row ----
-  if (active && !out_bytes) {  // packed nibbles [M][K/2]
+  if constexpr (!kA8) {
+  if (active && out_mode == 0) {  // packed nibbles [M][K/2]
     uint8_t* dst = xq + static_cast<size_t>(m) * (K / 2);
 #pragma unroll
     for (int run = 0; run < kEpt / kRun; ++run) {
@@ -346,8 +363,75 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
       }
     }
   }
+  }  // 4-bit
+  if constexpr (kA8) {
+    if (active) {
+#pragma unroll
+      for (int run = 0; run < kEpt / kRun; ++run) {
+        int e0;  // first element of this run within the row
+        if constexpr (kPhase2) {
+          e0 = ((j >> kR) << kLogB) | (run << kP) | ((j & ((1 << kR) - 1)) << kL);
+        } else {
+          e0 = j * kEpt;
+        }
+        if (out_mode == 2) {
+          // int8 codes [M][K], natural order
+          int8_t* dst = reinterpret_cast<int8_t*>(xq) + static_cast<size_t>(m) * K + e0;
+          if constexpr (kRun >= 8) {
+#pragma unroll
+            for (int t = 0; t < kRun / 8; ++t) {
+              const int w = run * (kRun / 8) + t;
+              *reinterpret_cast<uint2*>(dst + 8 * t) =
+                  make_uint2(__byte_perm(ev[w], od[w], 0x5140), __byte_perm(ev[w], od[w], 0x7362));
+            }
+          } else if constexpr (kRun == 4) {  // elements 4 h .. 4 h + 3 of group w
+            const int w = run >> 1, h = run & 1;
+            *reinterpret_cast<uint32_t*>(dst) = h ? __byte_perm(ev[w], od[w], 0x7362) : __byte_perm(ev[w], od[w], 0x5140);
+          } else {  // kRun == 2: elements 2 q, 2 q + 1 of group w
+            const int w = run >> 2, q = run & 3;
+            *reinterpret_cast<uint16_t*>(dst) =
+                static_cast<uint16_t>(((ev[w] >> (8 * q)) & 0xFFu) | (((od[w] >> (8 * q)) & 0xFFu) << 8));
+          }
+        } else {
+          // the GEMM's two operand planes [M][2K]: per k-block of 128 codes, 128 bytes of the
+          // high nibbles (E4M3 of v 2^-5) then 128 of the low nibbles (E4M3 of v 2^-9), each
+          // group of 8 in the order k0 k2 k4 k6 k1 k3 k5 k7; nibbles of q + 128
+          uint8_t* hp = xq + static_cast<size_t>(m) * (2 * K) + 2 * (e0 & ~127) + ((e0 & 127) & ~7);
+          uint8_t* lp = hp + 128;
+          auto planes = [&](int w, uint32_t& he, uint32_t& ho, uint32_t& le, uint32_t& lo) {
+            a8_planes(ev[w], od[w], he, ho, le, lo);
+          };
+          if constexpr (kRun >= 8) {
+#pragma unroll
+            for (int t = 0; t < kRun / 8; ++t) {
+              uint32_t he, ho, le, lo;
+              planes(run * (kRun / 8) + t, he, ho, le, lo);
+              *reinterpret_cast<uint2*>(hp + 8 * t) = make_uint2(he, ho);
+              *reinterpret_cast<uint2*>(lp + 8 * t) = make_uint2(le, lo);
+            }
+          } else if constexpr (kRun == 4) {  // elements o .. o + 3 (o = 4 h) of a group
+            const int w = run >> 1, h = run & 1, o = e0 & 7;
+            uint32_t he, ho, le, lo;
+            planes(w, he, ho, le, lo);
+            *reinterpret_cast<uint16_t*>(hp + (o >> 1)) = static_cast<uint16_t>(he >> (16 * h));
+            *reinterpret_cast<uint16_t*>(hp + 4 + (o >> 1)) = static_cast<uint16_t>(ho >> (16 * h));
+            *reinterpret_cast<uint16_t*>(lp + (o >> 1)) = static_cast<uint16_t>(le >> (16 * h));
+            *reinterpret_cast<uint16_t*>(lp + 4 + (o >> 1)) = static_cast<uint16_t>(lo >> (16 * h));
+          } else {  // kRun == 2: elements o, o + 1 (o = 2 q)
+            const int w = run >> 2, q = run & 3, o = e0 & 7;
+            uint32_t he, ho, le, lo;
+            planes(w, he, ho, le, lo);
+            hp[o >> 1] = static_cast<uint8_t>(he >> (8 * q));
+            hp[4 + (o >> 1)] = static_cast<uint8_t>(ho >> (8 * q));
+            lp[o >> 1] = static_cast<uint8_t>(le >> (8 * q));
+            lp[4 + (o >> 1)] = static_cast<uint8_t>(lo >> (8 * q));
+          }
+        }
+      }
+    }
+  }
   if (xsum != nullptr) {
-    int cs = static_cast<int>(sum_acc) - 8 * kEpt;  // every code carried an offset of 8
+    int cs = static_cast<int>(sum_acc) - (kA8 ? 128 : 8) * kEpt;  // every code carried an offset
     if ((tpr & 31) == 0) {
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) cs += __shfl_xor_sync(0xffffffffu, cs, o);
@@ -363,7 +447,7 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
   }
 }
 
-template <typename T, int kLogB, bool kStep>
+template <typename T, int kLogB, bool kStep, bool kA8>
 cudaError_t launch_t(const RotQuantArgs& a) {
   constexpr int kEpt = kLogB >= 12 ? 128 : 64;
   const int tpr = a.K / kEpt;
@@ -373,7 +457,7 @@ cudaError_t launch_t(const RotQuantArgs& a) {
   const int grid = (a.M + rows - 1) / rows;
   if (grid == 0) return cudaSuccess;
   const size_t smem = (kLogB > ((kEpt == 128) ? 7 : 6)) ? static_cast<size_t>(tpb) * kEpt * sizeof(float) : 0;
-  auto kern = rotate_quant_kernel<T, kLogB, kEpt, kStep>;
+  auto kern = rotate_quant_kernel<T, kLogB, kEpt, kStep, kA8>;
   if (smem > 48 * 1024) {
     // raise the kernel's limit once per device to the most any K asks of it (one kernel serves
     // several K, so several sizes: at most 256 threads x 128 float32 = 128 KB)
@@ -401,34 +485,35 @@ cudaError_t launch_t(const RotQuantArgs& a) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, reinterpret_cast<const T*>(a.x), a.M, a.K, a.inv_sqrt_b, a.step_scale,
-                                     a.xq, a.xscale, a.xsum, a.mode == 2 ? a.absmax : nullptr, a.out_bytes);
+                                     a.xq, a.xscale, a.xsum, a.mode == 2 ? a.absmax : nullptr, a.out_mode);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
-template <typename T, bool kStep>
+template <typename T, bool kStep, bool kA8>
 cudaError_t launch_mode(const RotQuantArgs& a) {
   switch (a.log_b) {
-    case 0: return launch_t<T, 0, kStep>(a);
-    case 1: return launch_t<T, 1, kStep>(a);
-    case 2: return launch_t<T, 2, kStep>(a);
-    case 3: return launch_t<T, 3, kStep>(a);
-    case 4: return launch_t<T, 4, kStep>(a);
-    case 5: return launch_t<T, 5, kStep>(a);
-    case 6: return launch_t<T, 6, kStep>(a);
-    case 7: return launch_t<T, 7, kStep>(a);
-    case 8: return launch_t<T, 8, kStep>(a);
-    case 9: return launch_t<T, 9, kStep>(a);
-    case 10: return launch_t<T, 10, kStep>(a);
-    case 11: return launch_t<T, 11, kStep>(a);
-    case 12: return launch_t<T, 12, kStep>(a);
+    case 0: return launch_t<T, 0, kStep, kA8>(a);
+    case 1: return launch_t<T, 1, kStep, kA8>(a);
+    case 2: return launch_t<T, 2, kStep, kA8>(a);
+    case 3: return launch_t<T, 3, kStep, kA8>(a);
+    case 4: return launch_t<T, 4, kStep, kA8>(a);
+    case 5: return launch_t<T, 5, kStep, kA8>(a);
+    case 6: return launch_t<T, 6, kStep, kA8>(a);
+    case 7: return launch_t<T, 7, kStep, kA8>(a);
+    case 8: return launch_t<T, 8, kStep, kA8>(a);
+    case 9: return launch_t<T, 9, kStep, kA8>(a);
+    case 10: return launch_t<T, 10, kStep, kA8>(a);
+    case 11: return launch_t<T, 11, kStep, kA8>(a);
+    case 12: return launch_t<T, 12, kStep, kA8>(a);
     default: return cudaErrorInvalidValue;
   }
 }
 
-template <typename T>
+// kA8: the 8-bit instantiations (out_mode 2 or 3), compiled in translation units of their own.
+template <typename T, bool kA8>
 cudaError_t launch_dtype(const RotQuantArgs& a) {
-  return a.mode == 1 ? launch_mode<T, true>(a) : launch_mode<T, false>(a);
+  return a.mode == 1 ? launch_mode<T, true, kA8>(a) : launch_mode<T, false, kA8>(a);
 }
 
 }  // namespace rq

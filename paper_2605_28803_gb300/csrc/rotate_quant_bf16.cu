@@ -2,5 +2,5 @@
 #include "rotate_quant.cuh"
 
 namespace qvla {
-cudaError_t launch_rotate_quant_bf16(const RotQuantArgs& a) { return rq::launch_dtype<__nv_bfloat16>(a); }
+cudaError_t launch_rotate_quant_bf16(const RotQuantArgs& a) { return rq::launch_dtype<__nv_bfloat16, false>(a); }
 }  // namespace qvla

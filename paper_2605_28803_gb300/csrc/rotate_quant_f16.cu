@@ -2,5 +2,5 @@
 #include "rotate_quant.cuh"
 
 namespace qvla {
-cudaError_t launch_rotate_quant_f16(const RotQuantArgs& a) { return rq::launch_dtype<__half>(a); }
+cudaError_t launch_rotate_quant_f16(const RotQuantArgs& a) { return rq::launch_dtype<__half, false>(a); }
 }  // namespace qvla

@@ -2,5 +2,5 @@
 #include "rotate_quant.cuh"
 
 namespace qvla {
-cudaError_t launch_rotate_quant_f32(const RotQuantArgs& a) { return rq::launch_dtype<float>(a); }
+cudaError_t launch_rotate_quant_f32(const RotQuantArgs& a) { return rq::launch_dtype<float, false>(a); }
 }  // namespace qvla

@@ -43,6 +43,10 @@ SIGNATURES = {
     "qvla_linear_quantize": (_I, [_P, _P, _I, _I, _P, _S, _P]),
     "qvla_linear_gemm": (_I, [_P, _P, _S, _I, _P, _P]),
     "qvla_w4a4_linear_noalloc": (_I, [_P, _P, _I, _I, _P, _P]),
+    "qvla_rotate_quantize_rows_a8": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
+    "qvla_w4a8_workspace_bytes": (_S, [_P, _I]),
+    "qvla_w4a8_linear": (_I, [_P, _P, _I, _I, _P, _P, _S, _P]),
+    "qvla_gemm_w4a8": (_I, [_P, _P, _P, _I, _P, _P, _P, _S, _P]),
     "qvla_check_device": (_I, [_P]),
 }
 
@@ -216,6 +220,26 @@ def qvla_w4a4_linear_noalloc(layer: Layer, x, M: int, step: int, y, stream=None)
     """qvla_w4a4_linear without a caller workspace: for callers that cannot allocate device
     memory while running; the library's fixed 8 MiB scratch takes the workspace's place."""
     _check(_lib.qvla_w4a4_linear_noalloc(layer.handle, _ptr(x), M, step, _ptr(y), _stream(stream)))
+
+
+def qvla_rotate_quantize_rows_a8(x, xdt: int, M: int, K: int, had_block: int, step_scale, xq, xscale, xsum=None,
+                                 stream=None) -> None:
+    _check(_lib.qvla_rotate_quantize_rows_a8(_ptr(x), xdt, M, K, had_block, _ptr(step_scale), _ptr(xq),
+                                             _ptr(xscale), _ptr(xsum), _stream(stream)))
+
+
+def qvla_w4a8_workspace_bytes(layer: Layer, M: int) -> int:
+    return int(_lib.qvla_w4a8_workspace_bytes(layer.handle, M))
+
+
+def qvla_w4a8_linear(layer: Layer, x, M: int, step: int, y, workspace, workspace_bytes: int, stream=None) -> None:
+    _check(_lib.qvla_w4a8_linear(layer.handle, _ptr(x), M, step, _ptr(y), _ptr(workspace), workspace_bytes,
+                                 _stream(stream)))
+
+
+def qvla_gemm_w4a8(layer: Layer, xq, xscale, M: int, y, acc, workspace, workspace_bytes: int, stream=None) -> None:
+    _check(_lib.qvla_gemm_w4a8(layer.handle, _ptr(xq), _ptr(xscale), M, _ptr(y), _ptr(acc), _ptr(workspace),
+                               workspace_bytes, _stream(stream)))
 
 
 def qvla_check_device(stream=None) -> None:
