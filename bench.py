@@ -19,7 +19,9 @@ The line also carries the two layer stacks (skipped with --no-stacks):
          down 4096 -> 1024) at M = 50 tokens with per-step scale tables, one CUDA graph per
          denoising step: microseconds per step (L2 flushed before each) and per 10-step rollout;
   "backbone": 18 layers of hidden 2048 with the gated 16384 MLP, per-token scales, one forward
-         pass at M = 816 (TOPS) and at M = 1 (HBM-bound: GB/s of packed weights).
+         pass at M = 816 (TOPS) and at M = 1 (HBM-bound: GB/s of packed weights);
+  "dit"."w4a8" and "w4a8_gate_up": the W4A8 variant (8-bit activation codes) on the DiT stack
+         and on the backbone's gate/up projection.
 """
 
 from __future__ import annotations
@@ -345,32 +347,15 @@ def _time_replays(fn, reps, flush=None, stream=None):
     return sum(a.elapsed_time(b) for a, b in evs) / reps
 
 
-def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
-    from paper_2605_28803_gb300 import qvla as Q
-    from paper_2605_28803_gb300 import stack as S
-    from paper_2605_28803_gb300 import workloads as W
-
-    scratch = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # 256 MB > 129 MB L2
-
-    def flush():
-        scratch.zero_()
-
-    # ---- DiT action head: per-step tables calibrated with the library's rotated-absmax pass ----
-    weights = W.dit_stack(DIT_SEED)
-    st = S.LinearStack(weights, DIT_M, "f16", "f16", dev, input_sets=DIT_T)
-    peak = torch.zeros(1, dtype=torch.float32, device=dev)
-    tables = []
+def _dit_stack(S, Q, W, weights, peaks, act_bits, dev, stream, flush, peak_gbs, peak_src):
+    """One DiT stack (18 blocks, M = 50, T = 10) with int4 or 8-bit activation codes: per-step
+    microseconds with L2 flushed, per rollout, and back to back."""
+    qmax = np.float32(7 if act_bits == 4 else 127)
+    st = S.LinearStack(weights, DIT_M, "f16", "f16", dev, input_sets=DIT_T, act_bits=act_bits)
     for i, w in enumerate(weights):
-        tab = []
-        for t in range(DIT_T):
-            xc = torch.from_numpy(W.dit_layer_input(DIT_SEED + 1000, i, t, DIT_CAL_ROWS, w.k, DIT_T)).to(dev, torch.float16)
-            peak.zero_()
-            Q.qvla_rotated_absmax(xc, Q.F16, DIT_CAL_ROWS, w.k, w.had_block, peak, stream)
-            tab.append(np.float32(peak.item()) / np.float32(7))
-        tables.append(np.asarray(tab, dtype=np.float32))
         for t in range(DIT_T):
             st.set_input(i, torch.from_numpy(W.dit_layer_input(DIT_SEED, i, t, DIT_M, w.k, DIT_T)), t)
-    st.set_step_tables(tables)
+    st.set_step_tables([p / qmax for p in peaks])
     graphs = [st.capture(t) for t in range(DIT_T)]
     for _ in range(3):
         for g in graphs:
@@ -384,7 +369,7 @@ def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
     Q.qvla_check_device(stream)
     dit_bytes = _algorithmic_bytes(weights, DIT_M)
     dit_gbs = dit_bytes / (step_ms * 1e-3) / 1e9
-    dit = {
+    out = {
         "us_per_step": round(step_ms * 1e3, 2), "us_per_rollout": round(roll_ms * 1e3, 2),
         "us_per_step_warm": round(warm_ms * 1e3, 2), "steps": DIT_T, "tokens": DIT_M,
         "linears_per_step": len(weights), "gpu_launches_per_step": 2 * len(weights),
@@ -394,11 +379,72 @@ def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
                      "peak_note": f"{peak_src} HBM copy bandwidth"},
         "timing": "CUDA-graph replay per step, L2 flushed (256 MB write) before each timed step or rollout; "
                   "'warm' = 10 steps back to back without a flush",
-        "tables": "per-step, per-layer, calibrated with qvla_rotated_absmax on a separate 16-token draw",
     }
     st.close()
     del graphs, st
     torch.cuda.empty_cache()
+    return out
+
+
+def _w4a8_gate_up(Q, W, dev, stream, flush, peak_tflops):
+    """The backbone's gate/up projection (816 x 2048 -> 2 x 16384, GELU-gated) with 8-bit
+    activation codes: rotate + quantise and the GEMM, TOPS of the integer product.  The tensor
+    cores run two E4M3 passes per product (high and low nibble planes), so the E4M3 rate the
+    hardware sustains is twice the reported TOPS."""
+    rng = np.random.default_rng(7)
+    codes = rng.integers(-7, 8, (2 * HIDDEN, K_IN)).astype(np.int8)
+    packed = W.pack_nibbles(codes)
+    ws = np.full(2 * HIDDEN, 2 ** -9, np.float32)
+    layer = Q.qvla_layer_create_gated(HIDDEN, K_IN, HAD_IN, Q.BF16, Q.BF16, packed[:HIDDEN], ws[:HIDDEN],
+                                      packed[HIDDEN:], ws[HIDDEN:])
+    x = torch.from_numpy(rng.standard_normal((M, K_IN), dtype=np.float32)).to(dev, torch.bfloat16)
+    h = torch.empty(M, HIDDEN, dtype=torch.bfloat16, device=dev)
+    nb = Q.qvla_w4a8_workspace_bytes(layer, M)
+    work = torch.empty(nb, dtype=torch.uint8, device=dev)
+
+    def run():
+        Q.qvla_w4a8_linear(layer, x, M, -1, h, work, nb, stream)
+
+    for _ in range(3):
+        run()
+    torch.cuda.synchronize()
+    Q.qvla_check_device(stream)
+    ms = _time_replays(run, 20, flush, stream)
+    Q.qvla_check_device(stream)
+    layer.close()
+    tops = OPS_GATEUP / (ms * 1e-3) / 1e12
+    return {"us": round(ms * 1e3, 1), "tops": round(tops, 1), "e4m3_tflops_issued": round(2 * tops, 1),
+            "frac_of_e4m3_peak": round(2 * tops / (FP8_OVER_BF16 * peak_tflops), 4),
+            "timing": "rotate+quantise (8-bit codes) and GEMM launches, L2 flushed before each of 20 runs"}
+
+
+def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
+    from paper_2605_28803_gb300 import qvla as Q
+    from paper_2605_28803_gb300 import stack as S
+    from paper_2605_28803_gb300 import workloads as W
+
+    scratch = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # 256 MB > 129 MB L2
+
+    def flush():
+        scratch.zero_()
+
+    # ---- DiT action head: per-step tables calibrated with the library's rotated-absmax pass ----
+    weights = W.dit_stack(DIT_SEED)
+    peak = torch.zeros(1, dtype=torch.float32, device=dev)
+    peaks = []  # [layer][step] rotated absmax of the calibration draw
+    for i, w in enumerate(weights):
+        row = []
+        for t in range(DIT_T):
+            xc = torch.from_numpy(W.dit_layer_input(DIT_SEED + 1000, i, t, DIT_CAL_ROWS, w.k, DIT_T)).to(dev, torch.float16)
+            peak.zero_()
+            Q.qvla_rotated_absmax(xc, Q.F16, DIT_CAL_ROWS, w.k, w.had_block, peak, stream)
+            row.append(np.float32(peak.item()))
+        peaks.append(np.asarray(row, dtype=np.float32))
+    dit = _dit_stack(S, Q, W, weights, peaks, 4, dev, stream, flush, peak_gbs, peak_src)
+    dit["w4a8"] = _dit_stack(S, Q, W, weights, peaks, 8, dev, stream, flush, peak_gbs, peak_src)
+    dit["tables"] = ("per-step, per-layer, calibrated with qvla_rotated_absmax on a separate 16-token draw "
+                     "(absmax / 7; absmax / 127 for the W4A8 variant)")
+    w4a8_gu = _w4a8_gate_up(Q, W, dev, stream, flush, peak_tflops)
 
     # ---- backbone forward at M = 816 and M = 1 (per-token scales) ----
     weights = W.backbone_stack(seed=3)
@@ -430,7 +476,7 @@ def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
     bb["timing"] = "CUDA-graph replay of one forward (2 kernels per linear), L2 flushed before each"
     del scratch
     torch.cuda.empty_cache()
-    return {"dit": dit, "backbone": bb}
+    return {"dit": dit, "backbone": bb, "w4a8_gate_up": w4a8_gu}
 
 
 # --------------------------------------------------------------------------------------

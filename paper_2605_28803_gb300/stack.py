@@ -2,8 +2,8 @@
 or of the DiT action head, each layer reading its own input buffer.
 
 Host-side plumbing only: every layer is one ``qvla_w4a4_linear`` call (the fused rotate +
-quantise kernel, then the GEMM with its dequantisation epilogue), so a stack of L linears is 2L
-kernel launches.  The kernels are launched with programmatic stream serialization, so
+quantise kernel, then the GEMM with its dequantisation epilogue), or ``qvla_w4a8_linear`` for
+8-bit activation codes, so a stack of L linears is 2L kernel launches.  The kernels are launched with programmatic stream serialization, so
 consecutive launches overlap their set-up with the previous kernel's tail; ``capture`` records
 a whole pass as a CUDA graph, which removes the host launch cost as well.  The per-step scale
 of a DiT layer is fixed at launch, so a DiT stack has one graph per denoising step.
@@ -28,8 +28,14 @@ class LinearStack:
     """Layers built from ``workloads.StackWeights``-like records (fields name, k, n,
     had_block, packed, wscale, bias, gated), all with m rows of input."""
 
-    def __init__(self, weights, m: int, xdtype: str = "f16", ydtype: str = "f16", device=None, input_sets: int = 1):
+    def __init__(self, weights, m: int, xdtype: str = "f16", ydtype: str = "f16", device=None, input_sets: int = 1,
+                 act_bits: int = 4):
+        if act_bits not in (4, 8):
+            raise ValueError("act_bits must be 4 or 8")
         self.m = m
+        self.act_bits = act_bits
+        self._linear = Q.qvla_w4a4_linear if act_bits == 4 else Q.qvla_w4a8_linear
+        ws_bytes = Q.qvla_linear_workspace_bytes if act_bits == 4 else Q.qvla_w4a8_workspace_bytes
         self.device = torch.device("cuda") if device is None else device
         xdt, self.xtorch = _DT[xdtype]
         ydt, self.ytorch = _DT[ydtype]
@@ -49,7 +55,7 @@ class LinearStack:
             for xs in self.sets:
                 xs.append(torch.zeros(m, w.k, dtype=self.xtorch, device=self.device))
             self.y.append(torch.empty(m, w.n, dtype=self.ytorch, device=self.device))
-        self.ws_bytes = max(Q.qvla_linear_workspace_bytes(layer, m) for layer in self.layers)
+        self.ws_bytes = max(ws_bytes(layer, m) for layer in self.layers)
         self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=self.device)
         self.weight_bytes = sum(int(w.packed.nbytes) for w in weights)
         self.ops = sum(2 * m * w.k * (2 * w.n if w.gated else w.n) for w in weights)
@@ -74,7 +80,7 @@ class LinearStack:
         """One pass over every layer; step -1 quantises per token, step t >= 0 with the tables."""
         stream = torch.cuda.current_stream() if stream is None else stream
         for layer, x, y in zip(self.layers, self.inputs(step), self.y):
-            Q.qvla_w4a4_linear(layer, x, self.m, step, y, self.ws, self.ws_bytes, stream)
+            self._linear(layer, x, self.m, step, y, self.ws, self.ws_bytes, stream)
 
     def capture(self, step: int = -1) -> torch.cuda.CUDAGraph:
         """A CUDA graph of one pass (2 kernels per layer), replayed with ``graph.replay()``."""

@@ -58,6 +58,36 @@ def test_dit_stack_every_linear_at_three_steps():
     assert clamped > 0, "the evaluation draw never exceeded the calibrated range"
 
 
+def test_dit_stack_w4a8_every_linear():
+    """The DiT stack with 8-bit activation codes (the appendix's W4A8 precision): per-step tables
+    of absmax / 127 from the same calibration draw, every linear checked at the first and last
+    step."""
+    weights = W.dit_stack(DIT_SEED)
+    tables = []
+    for i, w in enumerate(weights):
+        peaks = [O.robust_peak(O.rotate_activations(W.dit_layer_input(DIT_SEED + 1000, i, t, CAL_ROWS, w.k, DIT_T),
+                                                    w.had_block)) for t in range(DIT_T)]
+        tables.append(np.asarray(peaks, dtype=np.float32) / np.float32(127))
+    st = S.LinearStack(weights, DIT_M, "f16", "f16", G.DEV, act_bits=8)
+    st.set_step_tables(tables)
+    try:
+        for t in (0, DIT_T - 1):
+            for i, w in enumerate(weights):
+                st.set_input(i, torch.from_numpy(W.dit_layer_input(DIT_SEED, i, t, DIT_M, w.k, DIT_T)))
+            g = st.capture(t)
+            for y in st.y:
+                y.fill_(float("nan"))
+            g.replay()
+            torch.cuda.synchronize()
+            G.Q.qvla_check_device(G.stream())
+            for i, w in enumerate(weights):
+                ref = O.w4a4_linear(st.x[i].double().cpu().numpy(), w.codes, w.wscale, w.had_block, bias=w.bias,
+                                    table=tables[i], step=t, out_fmt="f16", act_bits=8)
+                G.assert_output_close(st.y[i].double().cpu().numpy(), ref["y"], "f16")
+    finally:
+        st.close()
+
+
 def _backbone_check(weights, st, rows, seed):
     """Sampled rows of every linear; all output channels of qkv and o, 256 of down, 128 hidden
     units (gate and up rows) of the gated layer.  The oracle unpacks the sampled weight rows."""
