@@ -101,6 +101,27 @@ qvla_status qvla_pack_weights_host(const void* W, qvla_dtype wdt, int N, int K,
 qvla_status qvla_block_svd_rotation(const void* W, qvla_dtype wdt, int N, int K, int block, int32_t* perm,
                                     double* rot);
 
+/* GPTQ-style weight codes (Sec. 5.1: the LLM side uses GPTQ with block size 128 and damping
+ * ratio 0.01; the appendix on weight-quantisation solvers), written from the published GPTQ
+ * algorithm.  Host only; a drop-in replacement of qvla_pack_weights_host's RTN codes with the
+ * same fold, scales and packed layout.
+ *   The weights are folded as in qvla_pack_weights_host and rounded to float32; Delta_W[n] is
+ *   the RTN scale max |W'_n| / 7.  The n_cal calibration rows X (host [n_cal][K], dtype xdt,
+ *   in the basis of W's input) are folded by the same P, U_b and Hadamard blocks, giving the
+ *   Hessian H = 2/n_cal X'^T X'.  A column with H_kk = 0 is dead (its codes are 0); H gets
+ *   damp * mean(diag H) on its diagonal.  With U the upper Cholesky factor of H^-1, the columns
+ *   are quantised in order, q = clamp(round(w_i / Delta), +-7), and the error
+ *   (w_i - Delta q) / U_ii is fed to every later column j times U_ij; updates beyond the current
+ *   block of `block` columns are applied once per block (block = 128 in the paper).
+ * Cost: O(K^3) for the factorisation and O(N K^2) for the codes (float64, all host cores);
+ * memory 2 K^2 doubles.  Returns QVLA_ERR_INVALID_ARG if the damped Hessian is not positive
+ * definite (e.g. damp = 0 with rank-deficient calibration data).
+ *   block >= 1, damp >= 0, n_cal >= 1, K <= 16384; other arguments as qvla_pack_weights_host. */
+qvla_status qvla_gptq_pack_host(const void* W, qvla_dtype wdt, int N, int K, const void* X, qvla_dtype xdt,
+                                int n_cal, const double* rot, int rot_block, const int32_t* perm,
+                                int had_block, int block, double damp, uint8_t* wq, float* wscale,
+                                int32_t* wsum);
+
 /* Upload already-packed weights as a layer (synchronous; allocates device memory the layer
  * owns).  wq host [N][K/2], wscale host [N], bias host [N] float32 or NULL.  xdt is the
  * activation dtype the layer accepts (F16, BF16 or F32); ydt the output dtype (F16 or BF16).

@@ -18,6 +18,9 @@ What is computed, in the paper's order (Sec. 4):
     DiT activation scales from a per-step table (Eq. 6, second display) looked up by t.
   * Sec. 4.2, Eq. 7: X'W' ~= Delta_X' Delta_W' Q_X' Q_W' (the integer GEMM and the
     dequantisation), plus the bias of the linear Y = XW + b (Sec. 3.2).
+  * Sec. 5.1 implementation details and the appendix on weight-quantisation solvers: the
+    LLM side's GPTQ-style weight codes (block size 128, damping ratio 0.01), written from
+    the published GPTQ algorithm the paper names.
 
 Precision.  Rotations, folds and the dequantised output are float64, rounded once
 to the output format.  Where floating point decides an integer (an int4 code) the
@@ -41,6 +44,10 @@ Readings of the paper that this file fixes (each is also listed in the design no
       keeps X W unchanged, R_hat^T P^T W.
   R15 U_b's columns are ordered by descending singular value, each signed so that its
       largest-magnitude entry is positive (the SVD fixes them only up to sign).
+  R17 GPTQ keeps the RTN per-channel scale (max |W'_n| / 7 of the folded weights) and
+      quantises the columns in natural order; its Hessian is H = 2/n X'^T X' of calibration
+      activations in the folded basis, damped by 0.01 mean(diag H); a column with
+      H_kk = 0 is dead (its weights become 0 and H_kk 1).
 
 Functions with no pin in the paper (the paper prints no worked numeric example) are
 pinned by closed forms, invariants, library special cases and brute force in
@@ -292,6 +299,62 @@ def quantize_weights(w_folded: np.ndarray):
     scale = absmax_scale(wf, axis=1)
     codes = quantize(wf, scale[:, None])
     return codes, scale
+
+
+def gptq_hessian(x_folded: np.ndarray) -> np.ndarray:
+    """H = 2/n X'^T X' (float64 [K, K]) of n calibration rows already in the folded basis
+    X' = X P R_hat: the Hessian of the layer-wise squared error ||X'W'^T - X'Q^T||^2 that GPTQ
+    minimises."""
+    x = np.asarray(x_folded, dtype=np.float64)
+    return (2.0 / x.shape[0]) * (x.T @ x)
+
+
+def gptq_quantize(w_folded: np.ndarray, h: np.ndarray, block: int = 128, damp: float = 0.01):
+    """GPTQ-style int4 weight codes (Sec. 5.1: the LLM side's solver, block size 128, damping
+    ratio 0.01), from the published GPTQ algorithm (reading R17):
+
+      1. scales as RTN: Delta_W[n] = float32(max |W'_n|) / 7 of the float32-rounded weights;
+      2. dead columns (H_kk = 0) are zeroed; H += damp * mean(diag H) * I;
+      3. U = the upper Cholesky factor of H^-1 (H^-1 = U^T U);
+      4. for each column i in order: q = clamp(round(w_i / Delta), +-7); the scaled error
+         e = (w_i - Delta q) / U_ii is subtracted, times U_ij, from every later column j;
+         within a block of `block` columns the later columns of the block are updated at
+         once, the columns after the block by one product at the end of the block.
+
+    w_folded: float64 [N, K]; h: float64 [K, K].  Returns (codes int8 [N, K], scales f32 [N]).
+    """
+    w = np.asarray(w_folded, dtype=np.float64).astype(np.float32).astype(np.float64)
+    n_rows, k = w.shape
+    scale = absmax_scale(w.astype(np.float32), axis=1)
+    d = scale.astype(np.float64)[:, None]
+    h = np.array(h, dtype=np.float64, copy=True)
+    dead = np.diag(h) == 0
+    h[dead, dead] = 1.0
+    w[:, dead] = 0.0
+    h[np.diag_indices(k)] += damp * np.mean(np.diag(h))
+    hinv = np.linalg.inv(h)
+    u = np.linalg.cholesky(hinv).T  # upper: hinv = u^T u
+    codes = np.zeros((n_rows, k), dtype=np.int8)
+    for i1 in range(0, k, block):
+        i2 = min(i1 + block, k)
+        err = np.zeros((n_rows, i2 - i1))
+        for i in range(i1, i2):
+            col = w[:, i]
+            with np.errstate(divide="ignore", invalid="ignore"):
+                t = np.where(d[:, 0] > 0, col / d[:, 0], 0.0)
+            q = np.clip(np.rint(t), -QMAX, QMAX)
+            codes[:, i] = q.astype(np.int8)
+            e = (col - d[:, 0] * q) / u[i, i]
+            w[:, i:i2] -= np.outer(e, u[i, i:i2])
+            err[:, i - i1] = e
+        w[:, i2:] -= err @ u[i1:i2, i2:]
+    return codes, scale
+
+
+def weight_proxy_loss(w_folded: np.ndarray, codes: np.ndarray, scale: np.ndarray, h: np.ndarray) -> float:
+    """tr((W' - Delta Q) H (W' - Delta Q)^T): the calibration error GPTQ reduces."""
+    dw = np.asarray(w_folded, dtype=np.float64) - np.asarray(scale, np.float64)[:, None] * codes
+    return float(np.einsum("nk,kl,nl->", dw, np.asarray(h, np.float64), dw))
 
 
 def pack_weights(w: np.ndarray, had_block: int, perm=None, rot=None, rot_block=None):

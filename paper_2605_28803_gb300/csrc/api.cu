@@ -153,6 +153,37 @@ qvla_status qvla_pack_weights_host(const void* W, qvla_dtype wdt, int N, int K, 
   return QVLA_OK;
 }
 
+qvla_status qvla_gptq_pack_host(const void* W, qvla_dtype wdt, int N, int K, const void* X, qvla_dtype xdt,
+                                int n_cal, const double* rot, int rot_block, const int32_t* perm, int had_block,
+                                int block, double damp, uint8_t* wq, float* wscale, int32_t* wsum) {
+  g_last_error.clear();
+  if (!W || !X || !wq || !wscale) return fail(QVLA_ERR_INVALID_ARG, "W, X, wq and wscale must not be NULL");
+  if (wdt != QVLA_F16 && wdt != QVLA_BF16 && wdt != QVLA_F32) return fail(QVLA_ERR_INVALID_ARG, "bad weight dtype %d", wdt);
+  if (xdt != QVLA_F16 && xdt != QVLA_BF16 && xdt != QVLA_F32) return fail(QVLA_ERR_INVALID_ARG, "bad calibration dtype %d", xdt);
+  if (qvla_status s = check_shape(N, K, had_block)) return s;
+  if (K > 16384) return fail(QVLA_ERR_INVALID_ARG, "K=%d: GPTQ supports K <= 16384", K);
+  if (n_cal < 1) return fail(QVLA_ERR_INVALID_ARG, "n_cal=%d must be >= 1", n_cal);
+  if (block < 1) return fail(QVLA_ERR_INVALID_ARG, "block=%d must be >= 1", block);
+  if (!(damp >= 0.0) || std::isinf(damp)) return fail(QVLA_ERR_INVALID_ARG, "damp must be finite and >= 0");
+  if (rot && (rot_block <= 0 || K % rot_block != 0))
+    return fail(QVLA_ERR_INVALID_ARG, "rot_block=%d must divide K=%d", rot_block, K);
+  if (perm) {
+    std::vector<char> seen(K, 0);
+    for (int k = 0; k < K; ++k) {
+      if (perm[k] < 0 || perm[k] >= K || seen[perm[k]]) return fail(QVLA_ERR_INVALID_ARG, "perm is not a permutation of [0, K)");
+      seen[perm[k]] = 1;
+    }
+  }
+  try {
+    if (!qvla::gptq_pack_host(W, static_cast<int>(wdt), N, K, X, static_cast<int>(xdt), n_cal, rot, rot_block, perm,
+                              had_block, block, damp, wq, wscale, wsum))
+      return fail(QVLA_ERR_INVALID_ARG, "the damped Hessian is not positive definite (raise damp)");
+  } catch (const std::bad_alloc&) {
+    return fail(QVLA_ERR_OOM, "host allocation failed");
+  }
+  return QVLA_OK;
+}
+
 qvla_status qvla_block_svd_rotation(const void* W, qvla_dtype wdt, int N, int K, int block, int32_t* perm,
                                     double* rot) {
   g_last_error.clear();

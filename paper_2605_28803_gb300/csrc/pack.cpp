@@ -7,6 +7,11 @@
 // Also the offline choice of P and U_b (Sec. 4.1, after Eq. 4): the zigzag channel permutation
 // by weight energy, and per block of input channels the left singular vectors of the block's
 // row partition, found as the eigenvectors of its Gram matrix by cyclic Jacobi rotations.
+//
+// And the LLM side's GPTQ-style codes (Sec. 5.1: block size 128, damping ratio 0.01), from the
+// published GPTQ algorithm: the RTN scale per output row, then the columns in order, each
+// column's rounding error fed forward through the upper Cholesky factor of the damped inverse
+// Hessian of calibration activations in the folded basis.
 #include "pack.h"
 
 #include <algorithm>
@@ -81,9 +86,10 @@ int quantize_code(float z, float d) {
   return static_cast<int>(r);
 }
 
-void pack_row(const void* W, int wdt, int K, int n, const double* rot, int rot_block, const int32_t* perm,
-              int had_block, std::vector<double>& a, std::vector<double>& b, std::vector<float>& f, uint8_t* wq,
-              float* wscale, int32_t* wsum) {
+// Row n of a [rows][K] matrix times P . BlockDiag(U_b) . BlockDiag(H_b / sqrt(b)) into a (float64);
+// b is scratch.  The same product folds a weight row (Eq. 5) and rotates an activation row.
+void fold_row(const void* W, int wdt, int K, int n, const double* rot, int rot_block, const int32_t* perm,
+              int had_block, std::vector<double>& a, std::vector<double>& b) {
   const size_t base = static_cast<size_t>(n) * K;
   for (int k = 0; k < K; ++k) a[k] = load_elem(W, wdt, base + (perm ? perm[k] : k));
   if (rot) {
@@ -109,6 +115,12 @@ void pack_row(const void* W, int wdt, int K, int n, const double* rot, int rot_b
       for (int i = 0; i < had_block; ++i) v[i] *= s;
     }
   }
+}
+
+void pack_row(const void* W, int wdt, int K, int n, const double* rot, int rot_block, const int32_t* perm,
+              int had_block, std::vector<double>& a, std::vector<double>& b, std::vector<float>& f, uint8_t* wq,
+              float* wscale, int32_t* wsum) {
+  fold_row(W, wdt, K, n, rot, rot_block, perm, had_block, a, b);
   float amax = 0.0f;
   for (int k = 0; k < K; ++k) {
     f[k] = static_cast<float>(a[k]);
@@ -265,6 +277,150 @@ void block_svd_rotation_host(const void* W, int wdt, int N, int K, int block, co
   for (unsigned i = 1; i < nt; ++i) pool.emplace_back(worker);
   worker();
   for (auto& t : pool) t.join();
+}
+
+namespace {
+
+// Runs fn(i) for i in [0, n) on up to 32 threads (contiguous chunks).
+template <typename F>
+void parallel_for(int n, F fn) {
+  if (n <= 0) return;
+  unsigned nt = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
+  nt = std::min<unsigned>(nt, static_cast<unsigned>(n));
+  if (nt == 1 || n < 64) {
+    for (int i = 0; i < n; ++i) fn(i);
+    return;
+  }
+  std::atomic<int> next{0};
+  auto worker = [&]() {
+    std::fesetround(FE_TONEAREST);
+    for (;;) {
+      const int i0 = next.fetch_add(16);
+      if (i0 >= n) break;
+      for (int i = i0; i < std::min(n, i0 + 16); ++i) fn(i);
+    }
+  };
+  std::vector<std::thread> pool;
+  for (unsigned t = 1; t < nt; ++t) pool.emplace_back(worker);
+  worker();
+  for (auto& t : pool) t.join();
+}
+
+}  // namespace
+
+bool gptq_pack_host(const void* W, int wdt, int N, int K, const void* X, int xdt, int n_cal, const double* rot,
+                    int rot_block, const int32_t* perm, int had_block, int block, double damp, uint8_t* wq,
+                    float* wscale, int32_t* wsum) {
+  std::fesetround(FE_TONEAREST);
+  const size_t KK = static_cast<size_t>(K) * K;
+  // calibration rows in the folded basis, stored transposed [K][n_cal] for the Hessian's dot products
+  std::vector<double> xt(static_cast<size_t>(K) * n_cal);
+  {
+    std::vector<double> a(K), b(K);
+    for (int r = 0; r < n_cal; ++r) {
+      fold_row(X, xdt, K, r, rot, rot_block, perm, had_block, a, b);
+      for (int k = 0; k < K; ++k) xt[static_cast<size_t>(k) * n_cal + r] = a[k];
+    }
+  }
+  // H = 2/n X'^T X' (both triangles)
+  std::vector<double> h(KK);
+  const double c2 = 2.0 / n_cal;
+  parallel_for(K, [&](int i) {
+    const double* xi = xt.data() + static_cast<size_t>(i) * n_cal;
+    for (int j = i; j < K; ++j) {
+      const double* xj = xt.data() + static_cast<size_t>(j) * n_cal;
+      double acc = 0.0;
+      for (int r = 0; r < n_cal; ++r) acc += xi[r] * xj[r];
+      h[static_cast<size_t>(i) * K + j] = c2 * acc;
+    }
+  });
+  for (int i = 0; i < K; ++i)
+    for (int j = 0; j < i; ++j) h[static_cast<size_t>(i) * K + j] = h[static_cast<size_t>(j) * K + i];
+  xt.clear();
+  xt.shrink_to_fit();
+  // dead columns and damping
+  std::vector<char> dead(K, 0);
+  double mean_diag = 0.0;
+  for (int k = 0; k < K; ++k) {
+    double& d = h[static_cast<size_t>(k) * K + k];
+    if (d == 0.0) {
+      dead[k] = 1;
+      d = 1.0;
+    }
+    mean_diag += d;
+  }
+  mean_diag /= K;
+  for (int k = 0; k < K; ++k) h[static_cast<size_t>(k) * K + k] += damp * mean_diag;
+  // H = T T^T with T upper triangular (Cholesky in reversed index order), in place in H's
+  // upper triangle; then U = T^-1 is upper triangular with H^-1 = U^T U, the factor GPTQ uses.
+  for (int j = K - 1; j >= 0; --j) {
+    double* hj = h.data() + static_cast<size_t>(j) * K;
+    double djj = hj[j];
+    for (int k = j + 1; k < K; ++k) djj -= hj[k] * hj[k];
+    if (!(djj > 0.0)) return false;
+    const double tjj = std::sqrt(djj);
+    hj[j] = tjj;
+    parallel_for(j, [&](int i) {
+      double* hi = h.data() + static_cast<size_t>(i) * K;
+      double v = hi[j];
+      for (int k = j + 1; k < K; ++k) v -= hi[k] * hj[k];
+      hi[j] = v / tjj;
+    });
+  }
+  std::vector<double> u(KK, 0.0);  // U = T^-1, column by column: T U[:, c] = e_c
+  parallel_for(K, [&](int c) {
+    u[static_cast<size_t>(c) * K + c] = 1.0 / h[static_cast<size_t>(c) * K + c];
+    for (int i = c - 1; i >= 0; --i) {
+      const double* hi = h.data() + static_cast<size_t>(i) * K;
+      double v = 0.0;
+      for (int k = i + 1; k <= c; ++k) v += hi[k] * u[static_cast<size_t>(k) * K + c];
+      u[static_cast<size_t>(i) * K + c] = -v / hi[i];
+    }
+  });
+  h.clear();
+  h.shrink_to_fit();
+  // each output row: the folded weights rounded to float32, the RTN scale, then the columns in
+  // order with error feedback; updates past the current block of columns are batched per block
+  parallel_for(N, [&](int n) {
+    std::vector<double> a(K), b(K), err(block);
+    fold_row(W, wdt, K, n, rot, rot_block, perm, had_block, a, b);
+    float amax = 0.0f;
+    for (int k = 0; k < K; ++k) {
+      const float f = static_cast<float>(a[k]);
+      a[k] = dead[k] ? 0.0 : static_cast<double>(f);
+      amax = std::max(amax, std::fabs(f));
+    }
+    const float d32 = amax / 7.0f;
+    const double d = d32;
+    wscale[n] = d32;
+    int32_t sum = 0;
+    uint8_t* row = wq + static_cast<size_t>(n) * (K / 2);
+    for (int i1 = 0; i1 < K; i1 += block) {
+      const int i2 = std::min(K, i1 + block);
+      for (int i = i1; i < i2; ++i) {
+        const double* ui = u.data() + static_cast<size_t>(i) * K;
+        double q = 0.0;
+        if (d > 0.0) q = std::min(7.0, std::max(-7.0, std::nearbyint(a[i] / d)));
+        const int qi = static_cast<int>(q);
+        sum += qi;
+        if (i & 1) {
+          row[i / 2] = static_cast<uint8_t>(row[i / 2] | ((qi & 0xF) << 4));
+        } else {
+          row[i / 2] = static_cast<uint8_t>(qi & 0xF);
+        }
+        const double e = (a[i] - d * q) / ui[i];
+        err[i - i1] = e;
+        for (int j = i; j < i2; ++j) a[j] -= e * ui[j];
+      }
+      for (int i = i1; i < i2; ++i) {
+        const double e = err[i - i1];
+        const double* ui = u.data() + static_cast<size_t>(i) * K;
+        for (int j = i2; j < K; ++j) a[j] -= e * ui[j];
+      }
+    }
+    if (wsum) wsum[n] = sum;
+  });
+  return true;
 }
 
 void code_sums_host(const uint8_t* wq, int N, int K, int32_t* wsum) {

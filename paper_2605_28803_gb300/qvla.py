@@ -28,6 +28,7 @@ SIGNATURES = {
     "qvla_abi_version": (_I, []),
     "qvla_pack_weights_host": (_I, [_P, _I, _I, _I, _P, _I, _P, _I, _P, _P, _P]),
     "qvla_block_svd_rotation": (_I, [_P, _I, _I, _I, _I, _P, _P]),
+    "qvla_gptq_pack_host": (_I, [_P, _I, _I, _I, _P, _I, _I, _P, _I, _P, _I, _I, _D, _P, _P, _P]),
     "qvla_layer_create": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, ctypes.POINTER(_P)]),
     "qvla_layer_create_gated": (_I, [_I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, ctypes.POINTER(_P)]),
     "qvla_pack_weights": (_I, [_P, _I, _I, _I, _P, _I, _P, _I, _P, _I, _I, ctypes.POINTER(_P)]),
@@ -104,6 +105,14 @@ def qvla_pack_weights_host(W: np.ndarray, wdt: int, N: int, K: int, rot=None, ro
     """Host-only fold + quantise + pack into caller-provided numpy buffers."""
     _check(_lib.qvla_pack_weights_host(_ptr(W), wdt, N, K, _ptr(rot), rot_block, _ptr(perm), had_block,
                                        _ptr(wq), _ptr(wscale), _ptr(wsum)))
+
+
+def qvla_gptq_pack_host(W: np.ndarray, wdt: int, N: int, K: int, X: np.ndarray, xdt: int, n_cal: int, rot=None,
+                        rot_block: int = 0, perm=None, had_block: int = 1, block: int = 128, damp: float = 0.01,
+                        wq=None, wscale=None, wsum=None) -> None:
+    """Host-only fold + GPTQ codes against calibration rows X + pack into caller-provided buffers."""
+    _check(_lib.qvla_gptq_pack_host(_ptr(W), wdt, N, K, _ptr(X), xdt, n_cal, _ptr(rot), rot_block, _ptr(perm),
+                                    had_block, block, float(damp), _ptr(wq), _ptr(wscale), _ptr(wsum)))
 
 
 def qvla_block_svd_rotation(W: np.ndarray, wdt: int, N: int, K: int, block: int):

@@ -396,6 +396,107 @@ def check_end_to_end_band(o):
     assert errs[512] < 0.7 * errs[1], errs
 
 
+def _correlated_calibration(rng, n, k, mix=0.6):
+    """Calibration rows with correlated channels: Z (I + mix A), Z and A Gaussian."""
+    a = rng.standard_normal((k, k)) / np.sqrt(k)
+    return rng.standard_normal((n, k)) @ (np.eye(k) + mix * a)
+
+
+def check_gptq_two_columns_closed_form(o):
+    """K = 2: after column 0 is rounded, column 1 absorbs its error d0 = w0 - Delta q0 as
+    w1 + d0 H01 / H11 (minimising the quadratic error over the free column), on the damped H."""
+    rng = np.random.default_rng(31)
+    for _ in range(20):
+        w = rng.standard_normal((5, 2))
+        x = _correlated_calibration(rng, 40, 2, mix=1.5)
+        h = o.gptq_hessian(x)
+        codes, scale = o.gptq_quantize(w, h, block=2, damp=0.01)
+        hd = h + 0.01 * np.mean(np.diag(h)) * np.eye(2)
+        w32 = w.astype(np.float32).astype(np.float64)
+        d = scale.astype(np.float64)
+        q0 = np.clip(np.rint(w32[:, 0] / d), -7, 7)
+        w1 = w32[:, 1] + (w32[:, 0] - d * q0) * hd[0, 1] / hd[1, 1]
+        q1 = np.clip(np.rint(w1 / d), -7, 7)
+        assert np.array_equal(codes[:, 0], q0) and np.array_equal(codes[:, 1], q1)
+
+
+def check_gptq_identity_hessian_is_rtn(o):
+    """With a diagonal Hessian no error crosses columns: GPTQ returns the RTN codes and scales."""
+    rng = np.random.default_rng(32)
+    w = rng.standard_normal((16, 64))
+    h = np.diag(rng.uniform(0.5, 2.0, 64))
+    codes, scale = o.gptq_quantize(w, h, block=16)
+    rc, rs = o.quantize_weights(w)
+    assert np.array_equal(scale, rs) and np.array_equal(codes, rc)
+
+
+def _obq_sequential(w, h, damp):
+    """The GPTQ result restated in the optimal-brain-quantiser form: one row at a time, column i
+    rounded, the remaining weights moved by -(w_i - Delta q_i) Hinv[i, :] / Hinv[i, i], and the
+    inverse Hessian updated by eliminating i (no Cholesky factor, no blocks)."""
+    w = np.asarray(w, dtype=np.float64).astype(np.float32).astype(np.float64)
+    k = w.shape[1]
+    hd = h + damp * np.mean(np.diag(h)) * np.eye(k)
+    out = np.zeros(w.shape, dtype=np.int8)
+    for n in range(w.shape[0]):
+        d = float(np.float32(np.abs(w[n].astype(np.float32)).max()) / np.float32(7))
+        row = w[n].copy()
+        hinv = np.linalg.inv(hd)
+        for i in range(k):
+            q = np.clip(np.rint(row[i] / d), -7, 7) if d > 0 else 0.0
+            out[n, i] = int(q)
+            row -= (row[i] - d * q) * hinv[i, :] / hinv[i, i]
+            hinv = hinv - np.outer(hinv[:, i], hinv[i, :]) / hinv[i, i]
+    return out
+
+
+def check_gptq_matches_obq_sequential(o):
+    """The Cholesky-and-blocks GPTQ equals the sequential OBQ elimination on small correlated
+    problems, for block sizes 1, 5 and K."""
+    rng = np.random.default_rng(33)
+    w = rng.standard_normal((6, 12)) * 0.1
+    h = o.gptq_hessian(_correlated_calibration(rng, 64, 12, mix=1.0))
+    ref = _obq_sequential(w, h, 0.01)
+    for block in (1, 5, 12):
+        codes, _ = o.gptq_quantize(w, h, block=block, damp=0.01)
+        assert np.array_equal(codes, ref), block
+
+
+def check_gptq_block_invariance_and_loss(o):
+    """Batching the updates in blocks does not change the result (block 1, 128, K), and on
+    correlated calibration data GPTQ's error tr(dW H dW^T) is below RTN's on every draw."""
+    rng = np.random.default_rng(34)
+    for seed in range(3):
+        r = np.random.default_rng(seed + 100)
+        x = o.block_hadamard_rotate(_correlated_calibration(r, 512, 256), 64)
+        w = o.block_hadamard_rotate(r.standard_normal((32, 256)) / 16.0, 64)
+        h = o.gptq_hessian(x)
+        c1, s1 = o.gptq_quantize(w, h, block=1)
+        c2, _ = o.gptq_quantize(w, h, block=128)
+        c3, _ = o.gptq_quantize(w, h, block=256)
+        assert np.array_equal(c1, c2) and np.array_equal(c1, c3)
+        rc, rs = o.quantize_weights(w)
+        assert np.array_equal(s1, rs)
+        lg = o.weight_proxy_loss(w, c1, s1, h)
+        lr = o.weight_proxy_loss(w, rc, rs, h)
+        assert lg < 0.9 * lr, (lg, lr)
+    del rng
+
+
+def check_gptq_dead_column(o):
+    """A calibration channel that is always zero leaves H_kk = 0: that column is dead, its codes
+    are 0, and the rest stays finite and within +-7."""
+    rng = np.random.default_rng(35)
+    x = _correlated_calibration(rng, 64, 32)
+    x[:, 5] = 0.0
+    w = rng.standard_normal((8, 32))
+    h = o.gptq_hessian(x)
+    h[5, :] = 0.0
+    h[:, 5] = 0.0
+    codes, scale = o.gptq_quantize(w, h)
+    assert np.all(codes[:, 5] == 0) and np.all(np.abs(codes) <= 7) and np.all(np.isfinite(scale))
+
+
 PINS = {f.__name__: f for f in [
     check_hadamard_matches_scipy, check_hadamard_orthogonal, check_hadamard_golden,
     check_rotate_matches_library_blockdiag, check_rotate_linf_bound, check_rotation_invariance,
@@ -405,6 +506,8 @@ PINS = {f.__name__: f for f in [
     check_weight_roundtrip, check_end_to_end_band,
     check_zigzag_golden, check_zigzag_rule, check_block_svd_golden, check_block_svd_properties,
     check_quantizer_8bit_bruteforce, check_w4a8_linear,
+    check_gptq_two_columns_closed_form, check_gptq_identity_hessian_is_rtn, check_gptq_matches_obq_sequential,
+    check_gptq_block_invariance_and_loss, check_gptq_dead_column,
 ]}
 
 
@@ -540,6 +643,36 @@ def _mut_svd_transposed(w, block, perm=None):
     return np.transpose(_real_block_svd(w, block, perm), (0, 2, 1)).copy()
 
 
+def _gptq_variant(sign=1.0, use_h=False, scale_err=True, tail=True):
+    """A GPTQ with one planted mistake (the oracle's steps otherwise)."""
+    def gptq(w_folded, h, block=128, damp=0.01):
+        w = np.asarray(w_folded, dtype=np.float64).astype(np.float32).astype(np.float64)
+        n_rows, k = w.shape
+        scale = O.absmax_scale(w.astype(np.float32), axis=1)
+        d = scale.astype(np.float64)
+        h = np.array(h, dtype=np.float64, copy=True)
+        dead = np.diag(h) == 0
+        h[dead, dead] = 1.0
+        w[:, dead] = 0.0
+        h[np.diag_indices(k)] += damp * np.mean(np.diag(h))
+        u = np.linalg.cholesky(h if use_h else np.linalg.inv(h)).T
+        codes = np.zeros((n_rows, k), dtype=np.int8)
+        for i1 in range(0, k, block):
+            i2 = min(i1 + block, k)
+            err = np.zeros((n_rows, i2 - i1))
+            for i in range(i1, i2):
+                col = w[:, i]
+                q = np.clip(np.rint(np.where(d > 0, col / np.where(d > 0, d, 1), 0.0)), -7, 7)
+                codes[:, i] = q.astype(np.int8)
+                e = (col - d * q) / (u[i, i] if scale_err else 1.0)
+                w[:, i:i2] -= sign * np.outer(e, u[i, i:i2])
+                err[:, i - i1] = e
+            if tail:
+                w[:, i2:] -= sign * (err @ u[i1:i2, i2:])
+        return codes, scale
+    return gptq
+
+
 MUTANTS = {
     "hadamard_wrong_order": ("sylvester_hadamard", _mut_hadamard_order),
     "rotate_unnormalised": ("block_hadamard_rotate", _mut_rotate_unnormalised),
@@ -560,6 +693,10 @@ MUTANTS = {
     "quantize_8bit_clamps_at_7": ("quantize", _mut_quantize_ignores_qmax),
     "svd_columns_ascending": ("block_svd_rotation", _mut_svd_ascending),
     "svd_factor_transposed_in_pack": ("block_svd_rotation", _mut_svd_transposed),
+    "gptq_update_sign_flipped": ("gptq_quantize", _gptq_variant(sign=-1.0)),
+    "gptq_cholesky_of_hessian": ("gptq_quantize", _gptq_variant(use_h=True)),
+    "gptq_error_not_scaled": ("gptq_quantize", _gptq_variant(scale_err=False)),
+    "gptq_no_update_past_block": ("gptq_quantize", _gptq_variant(tail=False)),
 }
 
 
