@@ -44,6 +44,9 @@ Readings of the paper that this file fixes (each is also listed in the design no
       keeps X W unchanged, R_hat^T P^T W.
   R15 U_b's columns are ordered by descending singular value, each signed so that its
       largest-magnitude entry is positive (the SVD fixes them only up to sign).
+  R18 The per-step table of Eq. 6 is also provided per channel group: one float32 per
+      (layer, step, group of max(128, b) channels) -- a k-block of the integer GEMM or a
+      Hadamard block; each group's integer partial is scaled by its Delta before the sum.
   R17 GPTQ keeps the RTN per-channel scale (max |W'_n| / 7 of the folded weights) and
       quantises the columns in natural order; its Hessian is H = 2/n X'^T X' of calibration
       activations in the folded basis, damped by 0.01 mean(diag H); a column with
@@ -393,6 +396,61 @@ def quantize_activations_per_step(y: np.ndarray, table, t: int, qmax: int = QMAX
     d = step_scale_lookup(table, t)
     scale = np.full(y.shape[0], d, dtype=np.float32)
     return quantize(y, scale[:, None], qmax), scale
+
+
+def step_group_size(k: int, had_block: int) -> int:
+    """Channels per scale of the per-step, per-group table (reading R18): max(128, b) -- one
+    128-channel k-block of the integer GEMM, or one Hadamard block when that is larger (after a
+    Hadamard block every channel of the block has the same spread, so a finer scale is moot)."""
+    g = max(128, had_block)
+    if k % g:
+        raise ValueError(f"K={k} is not a multiple of the group size {g}")
+    return g
+
+
+def quantize_activations_per_step_grouped(y: np.ndarray, table, t: int, group: int, qmax: int = QMAX):
+    """DiT activations with the per-step, per-group table of Eq. 6 (reading R18): channel k of
+    step t is quantised with table[t, k // group].  Returns (codes int8 [M, K], scales f32 [G])."""
+    table = np.asarray(table, dtype=np.float32)
+    if not (0 <= t < table.shape[0]):
+        raise IndexError(f"step {t} outside the table of {table.shape[0]} steps")
+    d = table[t]
+    if d.shape[0] * group != y.shape[1]:
+        raise ValueError("table width times group size must equal K")
+    per_channel = np.repeat(d, group)
+    return quantize(y, per_channel[None, :], qmax), d
+
+
+def grouped_linear(x: np.ndarray, w_codes: np.ndarray, w_scale: np.ndarray, had_block: int, table, step: int,
+                   bias=None, out_fmt: str = "f16", act_bits: int = 4):
+    """The online linear with per-step, per-group activation scales (Eq. 6 per channel group,
+    Eq. 7 per group): y = sum_g Delta_g Delta_W acc_g + b, where acc_g is the integer product
+    over group g's channels.  Float64 sum over the groups, rounded once to the output format."""
+    qmax = qmax_of(act_bits)
+    y32 = rotate_activations(x, had_block)
+    group = step_group_size(y32.shape[1], had_block)
+    qx, d = quantize_activations_per_step_grouped(y32, table, step, group, qmax)
+    n_groups = d.shape[0]
+    acc = [int_gemm(qx[:, g * group:(g + 1) * group], w_codes[:, g * group:(g + 1) * group]) for g in range(n_groups)]
+    y = np.zeros(acc[0].shape)
+    for g in range(n_groups):
+        y += np.float64(d[g]) * acc[g].astype(np.float64)
+    y = y * np.asarray(w_scale, dtype=np.float64)[None, :]
+    if bias is not None:
+        y = y + np.asarray(bias, dtype=np.float64)[None, :]
+    return {"y_rot": y32, "qx": qx, "dx": d, "acc_groups": acc, "y": round_to_format(y, out_fmt)}
+
+
+def calibrate_step_table_grouped(x_steps, had_block: int, estimator: str = "absmax", qmax: int = QMAX) -> np.ndarray:
+    """Per-step, per-group table [T, G] (reading R18): Delta_{t,g} = sigma_hat of group g's
+    channels of the rotated X_t, over q_max, float32."""
+    rows = []
+    for x in x_steps:
+        y = rotate_activations(x, had_block)
+        group = step_group_size(y.shape[1], had_block)
+        rows.append([np.float32(robust_peak(y[:, g * group:(g + 1) * group], estimator)) / np.float32(qmax)
+                     for g in range(y.shape[1] // group)])
+    return np.asarray(rows, dtype=np.float32)
 
 
 def robust_peak(y: np.ndarray, estimator: str = "absmax") -> np.float32:

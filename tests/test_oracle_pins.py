@@ -497,6 +497,61 @@ def check_gptq_dead_column(o):
     assert np.all(codes[:, 5] == 0) and np.all(np.abs(codes) <= 7) and np.all(np.isfinite(scale))
 
 
+def check_grouped_equal_scales_reduce_to_per_tensor(o):
+    """With every group of step t at the same scale the grouped linear is the per-tensor one."""
+    rng = np.random.default_rng(41)
+    x = rng.standard_normal((6, 512)) * 2.0
+    wc = rng.integers(-7, 8, (32, 512)).astype(np.int8)
+    ws = rng.uniform(0.01, 0.02, 32).astype(np.float32)
+    tab = np.array([0.3, 0.7], np.float32)
+    grouped = np.repeat(tab[:, None], 4, axis=1)
+    for t in range(2):
+        a = o.grouped_linear(x, wc, ws, 1, grouped, t, out_fmt="f32")["y"]
+        b = o.w4a4_linear(x, wc, ws, 1, table=tab, step=t, out_fmt="f32")["y"]
+        assert np.array_equal(a, b)
+
+
+def check_grouped_linear_bruteforce(o):
+    """Nested loops over m, n, k: y = sum_k Delta_{g(k)} q_x[m,k] q_w[n,k] Delta_W[n] + b, with
+    channel k in group k // max(128, b); codes by the nearest candidate per channel."""
+    rng = np.random.default_rng(42)
+    K, had = 256, 64
+    x = rng.standard_normal((3, K)) * 3.0
+    wc = rng.integers(-7, 8, (4, K)).astype(np.int8)
+    ws = rng.uniform(0.01, 0.02, 4).astype(np.float32)
+    bias = rng.standard_normal(4)
+    table = np.array([[0.2, 0.9], [1.3, 0.05]], np.float32)
+    out = o.grouped_linear(x, wc, ws, had, table, 1, bias=bias, out_fmt="f32")
+    y32 = o.rotate_activations(x, had)
+    for m in range(3):
+        for k in range(K):
+            d = float(table[1, k // 128])
+            t = float(y32[m, k]) / d
+            best = min(range(-7, 8), key=lambda q: (abs(t - q), q % 2))
+            assert out["qx"][m, k] == best
+    for m in range(3):
+        for n in range(4):
+            acc = sum(float(table[1, k // 128]) * int(out["qx"][m, k]) * int(wc[n, k]) for k in range(K))
+            ref = acc * float(ws[n]) + bias[n]
+            assert abs(out["y"][m, n] - ref) <= 2 ** -23 * max(1.0, abs(ref)), (m, n)
+
+
+def check_grouped_calibration(o):
+    """Each group's calibration peak maps to code +-7 exactly at its own scale; the group size is
+    max(128, b)."""
+    rng = np.random.default_rng(43)
+    xs = [rng.standard_normal((8, 512)) * (1.0 + t) * np.repeat(rng.uniform(0.5, 4.0, 4), 128)[None, :]
+          for t in range(3)]
+    tab = o.calibrate_step_table_grouped(xs, 64)
+    assert tab.shape == (3, 4)
+    assert o.step_group_size(512, 64) == 128 and o.step_group_size(4096, 1024) == 1024
+    for t in range(3):
+        y = o.rotate_activations(xs[t], 64)
+        q, _ = o.quantize_activations_per_step_grouped(y, tab, t, 128)
+        for g in range(4):
+            assert np.abs(q[:, g * 128:(g + 1) * 128]).max() == 7
+
+
 PINS = {f.__name__: f for f in [
     check_hadamard_matches_scipy, check_hadamard_orthogonal, check_hadamard_golden,
     check_rotate_matches_library_blockdiag, check_rotate_linf_bound, check_rotation_invariance,
@@ -508,6 +563,7 @@ PINS = {f.__name__: f for f in [
     check_quantizer_8bit_bruteforce, check_w4a8_linear,
     check_gptq_two_columns_closed_form, check_gptq_identity_hessian_is_rtn, check_gptq_matches_obq_sequential,
     check_gptq_block_invariance_and_loss, check_gptq_dead_column,
+    check_grouped_equal_scales_reduce_to_per_tensor, check_grouped_linear_bruteforce, check_grouped_calibration,
 ]}
 
 
@@ -673,6 +729,23 @@ def _gptq_variant(sign=1.0, use_h=False, scale_err=True, tail=True):
     return gptq
 
 
+def _mut_group_of_next_channel(y, table, t, group, qmax=7):
+    table = np.asarray(table, dtype=np.float32)
+    d = table[t]
+    per_channel = np.roll(np.repeat(d, group), 1)
+    return O.quantize(y, per_channel[None, :], qmax), d
+
+
+def _mut_group_first_only(y, table, t, group, qmax=7):
+    table = np.asarray(table, dtype=np.float32)
+    d = table[t]
+    return O.quantize(y, np.full((1, y.shape[1]), d[0], np.float32), qmax), d
+
+
+def _mut_group_size_fixed_128(k, had_block):
+    return 128
+
+
 MUTANTS = {
     "hadamard_wrong_order": ("sylvester_hadamard", _mut_hadamard_order),
     "rotate_unnormalised": ("block_hadamard_rotate", _mut_rotate_unnormalised),
@@ -697,6 +770,9 @@ MUTANTS = {
     "gptq_cholesky_of_hessian": ("gptq_quantize", _gptq_variant(use_h=True)),
     "gptq_error_not_scaled": ("gptq_quantize", _gptq_variant(scale_err=False)),
     "gptq_no_update_past_block": ("gptq_quantize", _gptq_variant(tail=False)),
+    "grouped_scale_shifted_one_channel": ("quantize_activations_per_step_grouped", _mut_group_of_next_channel),
+    "grouped_scale_first_group_only": ("quantize_activations_per_step_grouped", _mut_group_first_only),
+    "group_size_ignores_hadamard_block": ("step_group_size", _mut_group_size_fixed_128),
 }
 
 
