@@ -158,6 +158,21 @@ qvla_status qvla_layer_destroy(qvla_layer* layer);
  * Synchronous. */
 qvla_status qvla_set_step_scales(qvla_layer* layer, const float* scales, int T);
 
+/* Per-step, per-group activation scales (Eq. 6 read per channel group; reading: one float32
+ * per (step, group of max(128, had_block) channels) -- one k-block of the integer GEMM, or one
+ * Hadamard block when that is larger).  scales host [T][G] with G = K / group (see
+ * qvla_layer_scale_groups), each > 0 and finite.  Replaces any earlier table (per step or per
+ * group).  With such a table, qvla_w4a4_linear at step t quantises channel k with
+ * scales[t][k / group] and computes y = Delta_W[n] sum_g scales[t][g] acc_g[m,n] + bias[n],
+ * acc_g the exact integer product over group g's channels: each group's accumulator is
+ * corrected exactly and scaled before the float32 sum over the groups.  Not for gated layers
+ * (QVLA_ERR_UNSUPPORTED); the other step-taking entry points refuse grouped tables with
+ * QVLA_ERR_UNSUPPORTED (per-token calls, step == -1, are unaffected).  Synchronous. */
+qvla_status qvla_set_step_group_scales(qvla_layer* layer, const float* scales, int T, int G);
+
+/* The layer's scale groups: G groups of `group` channels (group = max(128, had_block)). */
+qvla_status qvla_layer_scale_groups(const qvla_layer* layer, int* G, int* group);
+
 /* Shape of a layer (N = output channels: H for a gated layer); any output pointer may be
  * NULL.  T is 0 when no table is set. */
 qvla_status qvla_layer_info(const qvla_layer* layer, int* N, int* K, int* had_block, int* T);
@@ -192,6 +207,12 @@ qvla_status qvla_rotate_quantize_rows(const void* x, qvla_dtype xdt, int M, int 
 qvla_status qvla_rotated_absmax(const void* x, qvla_dtype xdt, int M, int K, int had_block,
                                 float* absmax, void* stream);
 
+/* The same calibration per scale group: absmax device [K / group] floats (group =
+ * max(128, had_block), K a multiple of it), entry g raised to the max over the M rows and the
+ * group's channels.  The per-group table entry is then absmax[g] / 7. */
+qvla_status qvla_rotated_absmax_groups(const void* x, qvla_dtype xdt, int M, int K, int had_block,
+                                       float* absmax, void* stream);
+
 /* ------------------------------------------------------------------------------------------
  * Integer GEMM + dequantisation epilogue (Sec. 4.2 Eq. 7, scales "folded into
  * dequantization", Sec. 5.1):
@@ -209,7 +230,7 @@ qvla_status qvla_gemm_w4a4(const qvla_layer* layer, const uint8_t* xq, const flo
 
 /* Bytes of device workspace qvla_w4a4_linear needs for M rows (a multiple of 256): the codes
  * travel between its two kernels as one tensor-core operand byte each (M x K bytes), plus the
- * scales and code sums. */
+ * scales, the code sums and the per-group code sums (M x G x 4 bytes). */
 size_t qvla_linear_workspace_bytes(const qvla_layer* layer, int M);
 
 /* The whole online linear (Sec. 4): rotate + quantise x (as qvla_rotate_quantize, step as

@@ -1,6 +1,7 @@
 // The C ABI of libqvla (include/qvla.h): argument validation, layer objects and kernel dispatch.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -24,8 +25,11 @@ struct qvla_layer {
   float* wcorr = nullptr;     // device [N]: 8 * (sum of the codes of row n), the GEMM's offset correction
   float* wcorr8 = nullptr;    // device [N]: 128 * (sum of the codes of row n), the same for 8-bit activations
   float* bias = nullptr;      // device [N] (zeros when the layer was given none)
-  float* table = nullptr;     // device [table_cap]
+  float* table = nullptr;     // device [table_cap]: T step scales, or T x G group scales
   int T = 0, table_cap = 0;
+  int grouped = 0;            // the table holds one scale per (step, channel group)
+  int group = 128, G = 1;     // channels per scale group (max(128, had_block)) and groups per row
+  float* wgcorr = nullptr;    // device [N][G]: 8 * (sum of row n's codes over group g), non-gated layers
 };
 
 namespace {
@@ -93,7 +97,8 @@ qvla_status check_rows(int M) {
 }
 
 qvla_status launch_rq(const void* x, int xdt, int M, int K, int had_block, int mode, const float* step_scale,
-                      uint8_t* xq, float* xscale, int32_t* xsum, float* absmax, void* stream, int out_mode = 0) {
+                      uint8_t* xq, float* xscale, int32_t* xsum, float* absmax, void* stream, int out_mode = 0,
+                      int group = 0, int32_t* xgsum = nullptr) {
   qvla::RotQuantArgs a;
   a.x = x;
   a.xdt = xdt;
@@ -108,6 +113,8 @@ qvla_status launch_rq(const void* x, int xdt, int M, int K, int had_block, int m
   a.xsum = xsum;
   a.absmax = absmax;
   a.out_mode = out_mode;
+  a.gshift = group > 0 ? ilog2_exact(group) : 30;
+  a.xgsum = xgsum;
   a.stream = static_cast<cudaStream_t>(stream);
   QVLA_CUDA(qvla::launch_rotate_quant(a), "rotate_quantize launch");
   return QVLA_OK;
@@ -120,7 +127,7 @@ qvla_status resolve_step(const qvla_layer* layer, int step, const float** step_s
   }
   if (step < 0 || step >= layer->T)
     return fail(QVLA_ERR_STEP_RANGE, "step %d outside the layer's table of %d steps", step, layer->T);
-  *step_scale = layer->table + step;
+  *step_scale = layer->table + static_cast<size_t>(step) * (layer->grouped ? layer->G : 1);
   return QVLA_OK;
 }
 
@@ -223,6 +230,8 @@ static qvla_status upload_layer(int N, int K, int had_block, qvla_dtype xdt, qvl
   L->log_b = ilog2_exact(had_block);
   L->xdt = xdt;
   L->ydt = ydt;
+  L->group = std::max(128, had_block);
+  L->G = K / L->group;
   cudaGetDevice(&L->device);
   // Weights are stored tiled: each group of 128 rows x one k-block of 128 codes (64 bytes per
   // row) is one contiguous 8 KB chunk, chunks ordered by row group, then k-block; rows past N
@@ -252,6 +261,18 @@ static qvla_status upload_layer(int N, int K, int had_block, qvla_dtype xdt, qvl
   if (e == cudaSuccess) e = cudaMemcpy(L->wcorr, wcorr.data(), N * sizeof(float), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(L->wcorr8, wcorr8.data(), N * sizeof(float), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(L->bias, bias, N * sizeof(float), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !gated) {  // per-group code sums for per-group step scales
+    std::vector<float> wg(static_cast<size_t>(N) * L->G, 0.0f);
+    for (int n = 0; n < N; ++n)
+      for (int k = 0; k < K; ++k) {
+        const int b = wq[static_cast<size_t>(n) * rb + k / 2];
+        int q = (k & 1) ? (b >> 4) : (b & 0xF);
+        q = q >= 8 ? q - 16 : q;
+        wg[static_cast<size_t>(n) * L->G + k / L->group] += 8.0f * static_cast<float>(q);  // exact integers
+      }
+    e = cudaMalloc(&L->wgcorr, wg.size() * sizeof(float));
+    if (e == cudaSuccess) e = cudaMemcpy(L->wgcorr, wg.data(), wg.size() * sizeof(float), cudaMemcpyHostToDevice);
+  }
   if (e != cudaSuccess) {
     qvla_layer_destroy(L);
     return cuda_fail(e, "layer upload");
@@ -325,28 +346,65 @@ qvla_status qvla_layer_destroy(qvla_layer* L) {
   cudaFree(L->wscale);
   cudaFree(L->wcorr);
   cudaFree(L->wcorr8);
+  cudaFree(L->wgcorr);
   cudaFree(L->bias);
   cudaFree(L->table);
   delete L;
   return QVLA_OK;
 }
 
-qvla_status qvla_set_step_scales(qvla_layer* L, const float* scales, int T) {
-  g_last_error.clear();
-  if (!L || !scales) return fail(QVLA_ERR_INVALID_ARG, "layer and scales must not be NULL");
-  if (T < 1 || T > (1 << 20)) return fail(QVLA_ERR_INVALID_ARG, "T=%d must be in [1, 2^20]", T);
-  for (int t = 0; t < T; ++t)
-    if (!(scales[t] > 0.0f) || std::isinf(scales[t])) return fail(QVLA_ERR_INVALID_ARG, "scales[%d] must be finite and > 0", t);
-  if (T > L->table_cap) {  // grow; a smaller or equal table is written in place (graphs keep the address)
+namespace {
+qvla_status check_scales(const float* scales, size_t n) {
+  for (size_t i = 0; i < n; ++i)
+    if (!(scales[i] > 0.0f) || std::isinf(scales[i])) return fail(QVLA_ERR_INVALID_ARG, "scales[%zu] must be finite and > 0", i);
+  return QVLA_OK;
+}
+
+// Upload a table of T x per_step floats (already checked), growing the allocation only when it
+// is too small (a smaller or equal table is written in place: captured graphs keep the address).
+qvla_status upload_table(qvla_layer* L, const float* scales, int T, int per_step) {
+  const size_t n = static_cast<size_t>(T) * per_step;
+  L->T = 0;
+  if (n > static_cast<size_t>(L->table_cap)) {
     QVLA_CUDA(cudaDeviceSynchronize(), "synchronise before table reallocation");
     cudaFree(L->table);
     L->table = nullptr;
     L->table_cap = 0;
-    QVLA_CUDA(cudaMalloc(&L->table, T * sizeof(float)), "step table allocation");
-    L->table_cap = T;
+    QVLA_CUDA(cudaMalloc(&L->table, n * sizeof(float)), "step table allocation");
+    L->table_cap = static_cast<int>(n);
   }
-  QVLA_CUDA(cudaMemcpy(L->table, scales, T * sizeof(float), cudaMemcpyHostToDevice), "step table upload");
+  QVLA_CUDA(cudaMemcpy(L->table, scales, n * sizeof(float), cudaMemcpyHostToDevice), "step table upload");
   L->T = T;
+  return QVLA_OK;
+}
+}  // namespace
+
+qvla_status qvla_set_step_scales(qvla_layer* L, const float* scales, int T) {
+  g_last_error.clear();
+  if (!L || !scales) return fail(QVLA_ERR_INVALID_ARG, "layer and scales must not be NULL");
+  if (T < 1 || T > (1 << 20)) return fail(QVLA_ERR_INVALID_ARG, "T=%d must be in [1, 2^20]", T);
+  if (qvla_status s = check_scales(scales, static_cast<size_t>(T))) return s;
+  L->grouped = 0;
+  return upload_table(L, scales, T, 1);
+}
+
+qvla_status qvla_set_step_group_scales(qvla_layer* L, const float* scales, int T, int G) {
+  g_last_error.clear();
+  if (!L || !scales) return fail(QVLA_ERR_INVALID_ARG, "layer and scales must not be NULL");
+  if (L->gated) return fail(QVLA_ERR_UNSUPPORTED, "per-group step scales are not available for gated layers");
+  if (T < 1 || T > (1 << 16)) return fail(QVLA_ERR_INVALID_ARG, "T=%d must be in [1, 2^16]", T);
+  if (G != L->G)
+    return fail(QVLA_ERR_INVALID_ARG, "G=%d: this layer has %d groups of %d channels", G, L->G, L->group);
+  if (qvla_status s = check_scales(scales, static_cast<size_t>(T) * G)) return s;
+  L->grouped = 1;
+  return upload_table(L, scales, T, G);
+}
+
+qvla_status qvla_layer_scale_groups(const qvla_layer* L, int* G, int* group) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (G) *G = L->G;
+  if (group) *group = L->group;
   return QVLA_OK;
 }
 
@@ -379,6 +437,8 @@ qvla_status qvla_rotate_quantize(const qvla_layer* L, const void* x, int M, int 
   if (qvla_status s = check_rows(M)) return s;
   const float* ss = nullptr;
   if (qvla_status s = resolve_step(L, step, &ss)) return s;
+  if (ss && L->grouped)
+    return fail(QVLA_ERR_UNSUPPORTED, "per-group step scales run through qvla_w4a4_linear only (codes alone have no single scale)");
   if (M == 0) return QVLA_OK;
   if (!x || !xq || !xscale) return fail(QVLA_ERR_INVALID_ARG, "x, xq and xscale must not be NULL");
   if (!aligned16(x) || !aligned16(xq)) return fail(QVLA_ERR_INVALID_ARG, "x and xq must be 16-byte aligned");
@@ -394,6 +454,20 @@ qvla_status qvla_rotated_absmax(const void* x, qvla_dtype xdt, int M, int K, int
   if (!x || !absmax) return fail(QVLA_ERR_INVALID_ARG, "x and absmax must not be NULL");
   if (!aligned16(x)) return fail(QVLA_ERR_INVALID_ARG, "x must be 16-byte aligned");
   return launch_rq(x, xdt, M, K, had_block, 2, nullptr, nullptr, nullptr, nullptr, absmax, stream);
+}
+
+qvla_status qvla_rotated_absmax_groups(const void* x, qvla_dtype xdt, int M, int K, int had_block, float* absmax,
+                                       void* stream) {
+  g_last_error.clear();
+  if (qvla_status s = check_rows(M)) return s;
+  if (qvla_status s = check_shape(16, K, had_block)) return s;
+  if (xdt != QVLA_F16 && xdt != QVLA_BF16 && xdt != QVLA_F32) return fail(QVLA_ERR_INVALID_ARG, "bad activation dtype %d", xdt);
+  const int group = std::max(128, had_block);
+  if (K % group != 0) return fail(QVLA_ERR_INVALID_ARG, "K=%d is not a multiple of the group size %d", K, group);
+  if (M == 0) return QVLA_OK;
+  if (!x || !absmax) return fail(QVLA_ERR_INVALID_ARG, "x and absmax must not be NULL");
+  if (!aligned16(x)) return fail(QVLA_ERR_INVALID_ARG, "x must be 16-byte aligned");
+  return launch_rq(x, xdt, M, K, had_block, 2, nullptr, nullptr, nullptr, nullptr, absmax, stream, 0, group);
 }
 
 qvla_status qvla_rotate_quantize_rows_a8(const void* x, qvla_dtype xdt, int M, int K, int had_block,
@@ -414,7 +488,8 @@ qvla_status qvla_rotate_quantize_rows_a8(const void* x, qvla_dtype xdt, int M, i
 
 namespace {
 qvla_status launch_gemm(const qvla_layer* L, const uint8_t* xq, int x_bytes, const float* xscale, const int32_t* xsum,
-                        int M, void* y, int32_t* acc, void* stream) {
+                        int M, void* y, int32_t* acc, void* stream, const float* gscale = nullptr,
+                        const int32_t* xgsum = nullptr) {
   qvla::GemmArgs a;
   a.xq = xq;
   a.x_bytes = x_bytes;
@@ -431,6 +506,12 @@ qvla_status launch_gemm(const qvla_layer* L, const uint8_t* xq, int x_bytes, con
   a.N = L->N;
   a.K = L->K;
   a.gated = L->gated;
+  if (gscale) {
+    a.gscale = gscale;
+    a.xgsum = xgsum;
+    a.wgcorr = L->wgcorr;
+    a.group = L->group;
+  }
   a.num_sms = num_sms(L->device);
   a.stream = static_cast<cudaStream_t>(stream);
   QVLA_CUDA(qvla::launch_gemm_w4a4(a), "gemm launch");
@@ -454,8 +535,10 @@ qvla_status qvla_gemm_w4a4(const qvla_layer* L, const uint8_t* xq, const float* 
 
 size_t qvla_linear_workspace_bytes(const qvla_layer* L, int M) {
   if (!L || M <= 0) return 0;
-  // the codes travel between the two kernels as one operand byte each
-  return round256(static_cast<size_t>(M) * L->K) + round256(static_cast<size_t>(M) * 4) * 2;
+  // the codes travel between the two kernels as one operand byte each; then the scales, the
+  // code sums and the per-group code sums (used with per-group step scales)
+  return round256(static_cast<size_t>(M) * L->K) + round256(static_cast<size_t>(M) * 4) * 2 +
+         round256(static_cast<size_t>(M) * L->G * 4);
 }
 
 namespace {
@@ -463,6 +546,7 @@ struct LinearWorkspace {
   uint8_t* xb;       // [M][K] operand bytes
   float* xscale;     // [M]
   int32_t* xsum;     // [M]
+  int32_t* xgsum;    // [M][G]
 };
 
 qvla_status carve_workspace(const qvla_layer* L, int M, void* workspace, size_t workspace_bytes, LinearWorkspace* w) {
@@ -475,6 +559,7 @@ qvla_status carve_workspace(const qvla_layer* L, int M, void* workspace, size_t 
   w->xb = ws;
   w->xscale = reinterpret_cast<float*>(ws + round256(static_cast<size_t>(M) * L->K));
   w->xsum = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(w->xscale) + round256(static_cast<size_t>(M) * 4));
+  w->xgsum = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(w->xsum) + round256(static_cast<size_t>(M) * 4));
   return QVLA_OK;
 }
 }  // namespace
@@ -486,6 +571,8 @@ qvla_status qvla_linear_quantize(const qvla_layer* L, const void* x, int M, int 
   if (qvla_status s = check_rows(M)) return s;
   const float* ss = nullptr;
   if (qvla_status s = resolve_step(L, step, &ss)) return s;
+  if (ss && L->grouped)
+    return fail(QVLA_ERR_UNSUPPORTED, "per-group step scales run through qvla_w4a4_linear (the halves carry no step)");
   if (M == 0) return QVLA_OK;
   if (!x) return fail(QVLA_ERR_INVALID_ARG, "x must not be NULL");
   if (!aligned16(x)) return fail(QVLA_ERR_INVALID_ARG, "x must be 16-byte aligned");
@@ -519,6 +606,12 @@ qvla_status qvla_w4a4_linear(const qvla_layer* L, const void* x, int M, int step
   if (!aligned16(x) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "x and y must be 16-byte aligned");
   LinearWorkspace w;
   if (qvla_status s = carve_workspace(L, M, workspace, workspace_bytes, &w)) return s;
+  if (ss && L->grouped) {  // per-group step scales: per-group codes and sums, promoted per group
+    if (qvla_status s = launch_rq(x, L->xdt, M, L->K, L->had_block, 1, ss, w.xb, w.xscale, nullptr, nullptr, stream, 1,
+                                  L->group, w.xgsum))
+      return s;
+    return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream, ss, w.xgsum);
+  }
   if (qvla_status s = launch_rq(x, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr, stream, 1))
     return s;
   return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream);
@@ -571,6 +664,7 @@ qvla_status qvla_w4a8_linear(const qvla_layer* L, const void* x, int M, int step
   if (qvla_status s = check_rows(M)) return s;
   const float* ss = nullptr;
   if (qvla_status s = resolve_step(L, step, &ss)) return s;
+  if (ss && L->grouped) return fail(QVLA_ERR_UNSUPPORTED, "per-group step scales are for int4 activation codes");
   if (M == 0) return QVLA_OK;
   if (!x || !y) return fail(QVLA_ERR_INVALID_ARG, "x and y must not be NULL");
   if (!aligned16(x) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "x and y must be 16-byte aligned");

@@ -99,6 +99,14 @@ struct Params {
   int ldy;       // row length of y (N, or H for a gated layer)
   int splits;    // weight-major orientation: CTAs of a cluster splitting K (1 = no split)
   float kconst;  // the zero-point constant of the accumulator: 64 K (int4 codes), 1024 K (int8)
+  // per-group step scales (kGroup): the step's scales [ngroups], each group's code sums of the
+  // activations [M][ngroups] and 8 x of the weights [N][ngroups], k-blocks per group, 64 x
+  // the group's channels
+  const float* gscale;
+  const int32_t* xgsum;
+  const float* wgcorr;
+  int gkb, ngroups;
+  float gconst;
 };
 
 __device__ __forceinline__ void epi_sync() {
@@ -177,12 +185,18 @@ __device__ __forceinline__ void store_row32(OutT* dst, const uint32_t (&pk)[16],
 struct SplitParams {
   float cm, xs;       // kconst + 8 xsum[m], xscale[m]
   float4 wc, ws, bs;  // wcorr, wscale, bias of rows n .. n + 3
+  template <bool kGroup>
   __device__ __forceinline__ void load(const Params& p, int n, int m) {
     n = min(n, p.N - 4);
     m = min(m, p.M - 1);
-    cm = p.kconst + 8.0f * static_cast<float>(__ldg(p.xsum + m));
-    xs = __ldg(p.xscale + m);
-    wc = __ldg(reinterpret_cast<const float4*>(p.wcorr + n));
+    if constexpr (!kGroup) {  // grouped partials arrive scaled and corrected
+      cm = p.kconst + 8.0f * static_cast<float>(__ldg(p.xsum + m));
+      xs = __ldg(p.xscale + m);
+      wc = __ldg(reinterpret_cast<const float4*>(p.wcorr + n));
+    } else {
+      cm = xs = 0.0f;
+      wc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    }
     ws = __ldg(reinterpret_cast<const float4*>(p.wscale + n));
     bs = __ldg(reinterpret_cast<const float4*>(p.bias + n));
   }
@@ -193,7 +207,10 @@ struct SplitParams {
 // 128-byte swizzle straight into the MMA operand tile; only the weights are staged and
 // expanded.  2: the two operand planes of 8-bit codes ([rows][2K]: per k-block the high then
 // the low nibbles), both loaded per k-block and multiplied with the same expanded weight tile.
-template <int kBN, bool kSwap, bool kGated, int kX, typename OutT>
+// kGroup: per-step, per-group activation scales.  Each group's k-blocks accumulate into a fresh
+// TMEM buffer; the epilogue removes that group's zero point exactly, scales by the group's
+// Delta and adds the result into a running FP32 sum held in TMEM beside the two buffers.
+template <int kBN, bool kSwap, bool kGated, int kX, typename OutT, bool kGroup = false>
 __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_constant__ CUtensorMap tmap_a,
                                                                  const __grid_constant__ CUtensorMap tmap_b, Params p) {
   constexpr bool kXBytes = kX >= 1;
@@ -202,6 +219,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   constexpr bool kStageB = !(kXBytes && kSwap);
   using C = Cfg<kBN, kStageA, kStageB, kPlanes>;
   static_assert(kSwap || kBN % 128 == 0, "a weight tile is whole 128-row chunks");
+  static_assert(!kGroup || (kBN <= 128 && !kGated && kX == 1), "grouped scales: int4 operand bytes, BN <= 128");
+  // TMEM columns: two accumulators, plus the running sum of the grouped mode
+  constexpr uint32_t kTmemCols = !kGroup ? C::kTmemCols : (3 * kBN <= 64 ? 64 : 3 * kBN <= 128 ? 128 : 3 * kBN <= 256 ? 256 : 512);
   extern __shared__ uint8_t dyn_smem[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~uintptr_t(1023));
 
@@ -230,8 +250,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   // taking k-blocks [kb0, kb1); without a split every CTA runs whole tiles persistently
   const int splits = kSwap ? p.splits : 1;
   const uint32_t krank = (kSwap && splits > 1) ? cluster_ctarank() : 0u;
-  const int kb0 = (nkb_all * static_cast<int>(krank)) / splits;
-  const int kb1 = (nkb_all * (static_cast<int>(krank) + 1)) / splits;
+  // (grouped scales: the split falls on group boundaries, so each group's partial is whole)
+  const int kb0 = kGroup ? ((p.ngroups * static_cast<int>(krank)) / splits) * p.gkb
+                         : (nkb_all * static_cast<int>(krank)) / splits;
+  const int kb1 = kGroup ? ((p.ngroups * (static_cast<int>(krank) + 1)) / splits) * p.gkb
+                         : (nkb_all * (static_cast<int>(krank) + 1)) / splits;
   // this CTA's first tile and the tile stride, read where they are used (held in registers
   // across the role loops they would cost a register in every role)
 #define QVLA_UNIT0 (blockIdx.x / static_cast<unsigned>(splits))
@@ -253,7 +276,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     mbar_init_fence();
     s_epi_abort = 0;
   }
-  if (warp == kMmaWarp) tmem_alloc<C::kTmemCols>(smem_u32(&s_tmem_base));
+  if (warp == kMmaWarp) tmem_alloc<kTmemCols>(smem_u32(&s_tmem_base));
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -381,7 +404,37 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    if (lane == 0 && kGroup) {
+      // one accumulator per scale group, alternating between the two buffers group by group
+      constexpr uint32_t kIdesc = idesc_e4m3_f32(kBM, kBN);
+      int it = 0, gi = 0;
+      bool ok = true;
+      const int gkb = p.gkb;
+      for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS) {
+        for (int kg = kb0; kg < kb1; kg += gkb, ++gi) {
+          const int buf = gi & 1;
+          if (!mbar_wait(smem_u32(&bar_tempty[buf]), (static_cast<uint32_t>(gi >> 1) & 1u) ^ 1u)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t d = tmem_base + static_cast<uint32_t>(buf * kBN);
+          for (int q = 0; q < gkb; ++q, ++it) {
+            const int s = it % C::kStages;
+            const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
+            if (!mbar_wait(smem_u32(&bar_full[s]), ph)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t sa = smem_u32(smem + s * C::kStage);
+            const uint32_t sb = sa + C::kTileA;
+#pragma unroll
+            for (int kk = 0; kk < kBK / 32; ++kk)
+              mma_e4m3(d, smem_desc_sw128(sa + kk * 32), smem_desc_sw128(sb + kk * 32), kIdesc, (q != 0 || kk != 0) ? 1u : 0u);
+            mma_commit(smem_u32(&bar_empty[s]));
+          }
+          if (!ok) break;
+          mma_commit(smem_u32(&bar_tfull[buf]));
+        }
+      }
+      mma_commit(smem_u32(&bar_done));
+      mbar_wait(smem_u32(&bar_done), 0);
+    } else if (lane == 0) {
       constexpr uint32_t kIdesc = idesc_e4m3_f32(kBM, kBN);
       int it = 0, tile_iter = 0;
       bool ok = true;
@@ -425,6 +478,108 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     int tile_iter = 0;
     const float k64 = p.kconst;
     griddep_wait();  // xscale / xsum come from the previous kernel, and y may still be read by it
+    if constexpr (kGroup) {
+      // ---- grouped scales: promote each group's exact partial into the running sum ----
+      constexpr int kChunk = kBN < 32 ? kBN : 32;
+      const int G = p.ngroups, gkb = p.gkb;
+      const int g0 = kb0 / gkb, g1 = kb1 / gkb;
+      const float gconst = p.gconst;
+      int gi = 0;
+      for (int tile = QVLA_UNIT0; tile < ntiles; tile += QVLA_NUNITS) {
+        const int ta = tile % tiles_a, tb = tile / tiles_a;
+        epi_sync();
+        if (s_epi_abort) break;
+        if constexpr (!kSwap) {
+          for (int c = et; c < kBN; c += kEpiThreads) {
+            const int n = min(tb * kBN + c, p.N - 1);
+            s_ws[c] = __ldg(p.wscale + n);
+            s_bs[c] = __ldg(p.bias + n);
+          }
+          epi_sync();
+        }
+        const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+        const uint32_t run = lane_base + static_cast<uint32_t>(2 * kBN);  // the running sum's columns
+        const int ra = ta * kBM + et;  // this thread's MMA-A row
+        bool ok = true;
+        for (int g = g0; g < g1; ++g, ++gi) {
+          const int buf = gi & 1;
+          if (!mbar_wait(smem_u32(&bar_tfull[buf]), static_cast<uint32_t>(gi >> 1) & 1u)) {
+            s_epi_abort = 1;
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t part = lane_base + static_cast<uint32_t>(buf * kBN);
+          const float dg = __ldg(p.gscale + g);
+          const bool first = g == g0, last = g == g1 - 1;
+          // the fixed part of this row's correction: 8 x its code sum over the group + 64 x size
+          const bool rok = ra < (kSwap ? p.N : p.M);
+          const int rc = rok ? ra : 0;
+          const float rcorr = kSwap ? __ldg(p.wgcorr + static_cast<size_t>(rc) * G + g) + gconst
+                                    : 8.0f * static_cast<float>(__ldg(p.xgsum + static_cast<size_t>(rc) * G + g)) + gconst;
+#pragma unroll 1
+          for (int c0 = 0; c0 < kBN; c0 += kChunk) {
+            uint32_t r[32], R[32];
+            __syncwarp();
+            if constexpr (kChunk == 32) {
+              tmem_ld32(part + c0, r);
+              if (!first) tmem_ld32(run + c0, R);
+            } else {
+              tmem_ld16(part + c0, r);
+              if (!first) tmem_ld16(run + c0, R);
+            }
+            tmem_ld_wait();
+            const int col0 = tb * kBN + c0;  // first column (token when swapped, weight row else)
+#pragma unroll
+            for (int i = 0; i < kChunk; ++i) {
+              const int col = min(col0 + i, (kSwap ? p.M : p.N) - 1);
+              const float ccorr = kSwap ? 8.0f * static_cast<float>(__ldg(p.xgsum + static_cast<size_t>(col) * G + g))
+                                        : __ldg(p.wgcorr + static_cast<size_t>(col) * G + g);
+              // exact: the group's integer accumulator, below 2^24
+              const float acc = fmaf(__uint_as_float(r[i]), 262144.0f, -(rcorr + ccorr));
+              R[i] = __float_as_uint(fmaf(dg, acc, first ? 0.0f : __uint_as_float(R[i])));
+            }
+            if (!last) {
+              if constexpr (kChunk == 32) {
+                tmem_st32(run + c0, R);
+              } else {
+                tmem_st16(run + c0, R);
+              }
+              continue;
+            }
+            // the last group: y = Delta_W[n] x (sum over groups) + bias
+            if constexpr (kSwap) {
+              const int n = ra;
+              if (splits > 1) {  // the cluster reduction below applies the epilogue
+                float* partial = reinterpret_cast<float*>(smem);
+#pragma unroll
+                for (int i = 0; i < kChunk; ++i) partial[(c0 + i) * kBM + et] = __uint_as_float(R[i]);
+              } else if (rok) {
+                const float ws = __ldg(p.wscale + n), b = __ldg(p.bias + n);
+#pragma unroll
+                for (int i = 0; i < kChunk; ++i) {
+                  const int m = col0 + i;
+                  if (m < p.M)
+                    reinterpret_cast<OutT*>(p.y)[static_cast<size_t>(m) * p.ldy + n] =
+                        to_out<OutT>(fmaf(__uint_as_float(R[i]), ws, b));
+                }
+              }
+            } else if (rok && col0 < p.N) {
+              uint32_t pk[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i)
+                pk[i] = pack2<OutT>(fmaf(__uint_as_float(R[2 * i]), s_ws[c0 + 2 * i], s_bs[c0 + 2 * i]),
+                                    fmaf(__uint_as_float(R[2 * i + 1]), s_ws[c0 + 2 * i + 1], s_bs[c0 + 2 * i + 1]));
+              store_row32(reinterpret_cast<OutT*>(p.y) + static_cast<size_t>(ra) * p.ldy + col0, pk, min(32, p.N - col0));
+            }
+          }
+          tmem_st_wait();
+          tc_fence_before();
+          mbar_arrive(smem_u32(&bar_tempty[buf]));
+        }
+        if (!ok) continue;
+      }
+    } else
     for (int tile = QVLA_UNIT0; tile < ntiles; tile += QVLA_NUNITS, ++tile_iter) {
       const int ta = tile % tiles_a, tb = tile / tiles_a;
       const int buf = tile_iter & 1;
@@ -623,7 +778,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       if (e < total) {
         int n, m, row, col;
         coords(e, n, m, row, col);
-        nxt.load(p, n, m);
+        nxt.template load<kGroup>(p, n, m);
       }
       cluster_wait();
       const uint32_t part0 = smem_u32(smem);
@@ -634,7 +789,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
         if (e + kThreads < total) {
           int n2, m2, r2, c2;
           coords(e + kThreads, n2, m2, r2, c2);
-          nxt.load(p, n2, m2);
+          nxt.template load<kGroup>(p, n2, m2);
         }
         const uint32_t off = static_cast<uint32_t>((col * kBM + row) * 4);
         float4 v[8];
@@ -651,7 +806,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
             sum.z += v[q].z;
             sum.w += v[q].w;
           }
-        if (n < p.N && m < p.M) {  // N % 16 == 0, so rows n .. n + 3 all exist
+        if (kGroup && n < p.N && m < p.M) {  // grouped: the partials are scaled and corrected sums
+          const uint32_t lo = pack2<OutT>(fmaf(sum.x, cur.ws.x, cur.bs.x), fmaf(sum.y, cur.ws.y, cur.bs.y));
+          const uint32_t hi = pack2<OutT>(fmaf(sum.z, cur.ws.z, cur.bs.z), fmaf(sum.w, cur.ws.w, cur.bs.w));
+          *reinterpret_cast<uint2*>(reinterpret_cast<OutT*>(p.y) + static_cast<size_t>(m) * p.ldy + n) =
+              make_uint2(lo, hi);
+        } else if (n < p.N && m < p.M) {  // N % 16 == 0, so rows n .. n + 3 all exist
           const float a0 = fmaf(sum.x, 262144.0f, -(cur.wc.x + cur.cm));
           const float a1 = fmaf(sum.y, 262144.0f, -(cur.wc.y + cur.cm));
           const float a2 = fmaf(sum.z, 262144.0f, -(cur.wc.z + cur.cm));
@@ -671,7 +831,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     }
   }
   tc_fence_after();
-  if (warp == kMmaWarp) tmem_dealloc<C::kTmemCols>(tmem_base);
+  if (warp == kMmaWarp) tmem_dealloc<kTmemCols>(tmem_base);
 #undef QVLA_UNIT0
 #undef QVLA_NUNITS
 }
@@ -753,7 +913,7 @@ int max_active_clusters(const void* kern, const cudaLaunchConfig_t& cfg) {
   return n;
 }
 
-template <int kBN, bool kSwap, bool kGated, int kX, typename OutT>
+template <int kBN, bool kSwap, bool kGated, int kX, typename OutT, bool kGroup = false>
 cudaError_t launch_cfg(const GemmArgs& a) {
   constexpr bool kXBytes = kX >= 1;
   constexpr int kPlanes = kX == 2 ? 2 : 1;
@@ -774,6 +934,12 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   }
   p.K = a.K;
   p.kconst = (kX == 2 ? 1024.0f : 64.0f) * static_cast<float>(a.K);
+  p.gscale = a.gscale;
+  p.xgsum = a.xgsum;
+  p.wgcorr = a.wgcorr;
+  p.gkb = a.group / kBK;
+  p.ngroups = a.group > 0 ? a.K / a.group : 0;
+  p.gconst = 64.0f * static_cast<float>(a.group);
   p.xscale = a.xscale;
   p.xsum = a.xsum;
   p.wscale = a.wscale;
@@ -786,7 +952,7 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   p.ldy = a.gated ? a.N / 2 : a.N;
   const int tiles = ((p.rows_a + kBM - 1) / kBM) * ((p.rows_b + kBN - 1) / kBN);
   if (tiles == 0) return cudaSuccess;
-  auto kern = gemm_w4a4_kernel<kBN, kSwap, kGated, kX, OutT>;
+  auto kern = gemm_w4a4_kernel<kBN, kSwap, kGated, kX, OutT, kGroup>;
   cudaError_t e = prepare_kernel(reinterpret_cast<const void*>(kern), C::kSmem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -806,7 +972,7 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   // up to 8 CTAs, as long as every cluster of the grid can be resident at once
   int splits = 1;
   if (kSwap) {
-    const int nkb = p.K / kBK;
+    const int nkb = kGroup ? p.ngroups : p.K / kBK;  // grouped scales split whole groups
     while (splits < 8 && 2 * splits <= nkb && tiles * 2 * splits <= a.num_sms) {
       attr[1].val.clusterDim.x = static_cast<unsigned>(2 * splits);
       cfg.gridDim = dim3(tiles * 2 * splits);
@@ -834,6 +1000,19 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   return cudaGetLastError();
 }
 
+// Per-group step scales: int4 operand bytes, 128-wide tiles at most (the running sum takes a
+// third TMEM region).
+template <typename OutT>
+cudaError_t launch_grouped(const GemmArgs& a) {
+  if (a.gated || a.x_bytes != 1) return cudaErrorInvalidValue;
+  if (a.M > 128) return launch_cfg<128, false, false, 1, OutT, true>(a);
+  const int mpad = (a.M + 15) / 16 * 16;
+  if (mpad <= 16) return launch_cfg<16, true, false, 1, OutT, true>(a);
+  if (mpad <= 32) return launch_cfg<32, true, false, 1, OutT, true>(a);
+  if (mpad <= 64) return launch_cfg<64, true, false, 1, OutT, true>(a);
+  return launch_cfg<128, true, false, 1, OutT, true>(a);
+}
+
 template <int kX, typename OutT>
 cudaError_t launch_out(const GemmArgs& a) {
   if (a.gated) return launch_cfg<256, false, true, kX, OutT>(a);  // gate/up pairs share a 256-row tile
@@ -857,6 +1036,7 @@ cudaError_t launch_out(const GemmArgs& a) {
 
 cudaError_t launch_gemm_w4a4(const GemmArgs& a) {
   if (a.M == 0) return cudaSuccess;
+  if (a.gscale) return a.ydt == 0 ? launch_grouped<__half>(a) : launch_grouped<__nv_bfloat16>(a);
   if (a.x_bytes == 2) return a.ydt == 0 ? launch_out<2, __half>(a) : launch_out<2, __nv_bfloat16>(a);
   if (a.x_bytes == 1) return a.ydt == 0 ? launch_out<1, __half>(a) : launch_out<1, __nv_bfloat16>(a);
   return a.ydt == 0 ? launch_out<0, __half>(a) : launch_out<0, __nv_bfloat16>(a);

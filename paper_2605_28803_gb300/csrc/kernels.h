@@ -24,7 +24,11 @@ struct RotQuantArgs {
                            //   [M][2K] (per 128 codes: high nibbles, then low nibbles)
   float* xscale;           // device [M]
   int32_t* xsum;           // device [M] or null
-  float* absmax;           // device, one float (mode 2)
+  float* absmax;           // device, one float (mode 2), or one per scale group
+  int gshift = 30;         // scale groups of 2^gshift channels (>= 30: one group; else a group
+                           //   holds whole Hadamard blocks and >= 128 channels): step_scale
+                           //   then points at the step's [K >> gshift] entries, absmax too
+  int32_t* xgsum = nullptr;  // device [M][K >> gshift] per-group code sums, or null
   cudaStream_t stream;
 };
 bool rotate_quant_supported(int log_b);
@@ -53,6 +57,13 @@ struct GemmArgs {
   int32_t* acc;            // device [M][N] or null
   int M, N, K;             // N = weight rows (2H for a gated layer)
   int gated;               // 1: rows interleave gate/up in 128-row groups; y is [M][N/2] = h
+  // per-step, per-group activation scales (x_bytes 1, not gated; acc unused): gscale device
+  // [K/group] the step's scales, xgsum device [M][K/group] the activations' group code sums,
+  // wgcorr device [N][K/group] 8 x the weights' group code sums; group = channels per scale
+  const float* gscale = nullptr;
+  const int32_t* xgsum = nullptr;
+  const float* wgcorr = nullptr;
+  int group = 0;
   int num_sms;
   cudaStream_t stream;
 };

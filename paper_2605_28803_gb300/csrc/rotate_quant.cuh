@@ -129,14 +129,19 @@ __device__ __forceinline__ uint32_t sum8_offset(uint32_t w, uint32_t acc) {
 
 // kLogB: log2 of the Hadamard block (0 = no rotation).  kEpt: elements per thread.
 // kStep: the scale is the step table entry (else per token; per-token mode also serves the
-// calibration max when absmax_out is set).  kA8: 8-bit codes (q_max 127; out_mode int8 rows
-// or the GEMM's two operand planes), else 4-bit (q_max 7; packed nibbles or operand bytes).
+// calibration max when absmax_out is set).  Scale groups: channel k belongs to group
+// k >> gshift (gshift >= 30: one group).  A group holds whole Hadamard blocks and at least 128
+// channels, so all of a thread's elements share one group: with a per-group step table
+// (step_scale[g]) the thread takes its group's entry, xgsum (when set) receives each group's
+// code sum [M][K >> gshift], and calibration (absmax_out) raises one maximum per group.
+// kA8: 8-bit codes (q_max 127; out_mode int8 rows or the GEMM's two operand planes), else
+// 4-bit (q_max 7; packed nibbles or operand bytes).
 template <typename T, int kLogB, int kEpt, bool kStep, bool kA8>
 __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__ x, int M, int K, float inv_sqrt_b,
                                                              const float* __restrict__ step_scale,
                                                              uint8_t* __restrict__ xq, float* __restrict__ xscale,
                                                              int32_t* __restrict__ xsum, float* __restrict__ absmax_out,
-                                                             int out_mode) {
+                                                             int out_mode, int gshift, int32_t* __restrict__ xgsum) {
   constexpr float kQ = kA8 ? 127.0f : 7.0f;
   constexpr float kBand = kA8 ? kTieBand8 : kTieBand;
   constexpr int kP = (kEpt == 128) ? 7 : 6;  // log2(kEpt)
@@ -160,6 +165,14 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
   const int j = tid - rloc * tpr;     // thread within the row
   const int m = blockIdx.x * rpc + rloc;
   const bool active = (rloc < rpc) && (m < M);
+  // the channel of this thread's first element, and so its scale group
+  int e_first;
+  if constexpr (kPhase2) {
+    e_first = ((j >> kR) << kLogB) | ((j & ((1 << kR) - 1)) << kL);
+  } else {
+    e_first = j * kEpt;
+  }
+  const int grp = gshift >= 30 ? 0 : e_first >> gshift;
 
   if (tid < 32) {
     s_max[tid] = 0u;
@@ -218,11 +231,19 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
   // ---- scale ----
   float delta;
   if constexpr (kStep) {
-    delta = __ldg(step_scale);
+    delta = __ldg(step_scale + grp);
   } else {
     float w = 0.0f;
 #pragma unroll
     for (int i = 0; i < kN; ++i) w = fmaxf(w, fmaxf(fabsf(v[i].x), fabsf(v[i].y)));
+    if (absmax_out != nullptr && gshift < 30) {
+      // per-group calibration: the group's threads are consecutive lanes, tg of them (tg | 32)
+      const int tg = (1 << gshift) / kEpt;
+      for (int o = tg >> 1; o > 0; o >>= 1) w = fmaxf(w, __shfl_xor_sync(0xffffffffu, w, o));
+      if (active && (j & (tg - 1)) == 0)
+        atomicMax(reinterpret_cast<unsigned int*>(absmax_out + grp), __float_as_uint(w * inv_sqrt_b));
+      return;
+    }
     if ((tpr & 31) == 0) {
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) w = fmaxf(w, __shfl_xor_sync(0xffffffffu, w, o));
@@ -430,6 +451,12 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
       }
     }
   }
+  if (xgsum != nullptr) {  // the code sum of each scale group of the row (tg consecutive lanes)
+    int gs = static_cast<int>(sum_acc) - (kA8 ? 128 : 8) * kEpt;
+    const int tg = (1 << gshift) / kEpt;
+    for (int o = tg >> 1; o > 0; o >>= 1) gs += __shfl_xor_sync(0xffffffffu, gs, o);
+    if (active && (j & (tg - 1)) == 0) xgsum[static_cast<size_t>(m) * (K >> gshift) + grp] = gs;
+  }
   if (xsum != nullptr) {
     int cs = static_cast<int>(sum_acc) - (kA8 ? 128 : 8) * kEpt;  // every code carried an offset
     if ((tpr & 31) == 0) {
@@ -485,7 +512,8 @@ cudaError_t launch_t(const RotQuantArgs& a) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, reinterpret_cast<const T*>(a.x), a.M, a.K, a.inv_sqrt_b, a.step_scale,
-                                     a.xq, a.xscale, a.xsum, a.mode == 2 ? a.absmax : nullptr, a.out_mode);
+                                     a.xq, a.xscale, a.xsum, a.mode == 2 ? a.absmax : nullptr, a.out_mode,
+                                     a.gshift, a.xgsum);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

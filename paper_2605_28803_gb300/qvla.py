@@ -34,6 +34,9 @@ SIGNATURES = {
     "qvla_pack_weights": (_I, [_P, _I, _I, _I, _P, _I, _P, _I, _P, _I, _I, ctypes.POINTER(_P)]),
     "qvla_layer_destroy": (_I, [_P]),
     "qvla_set_step_scales": (_I, [_P, _P, _I]),
+    "qvla_set_step_group_scales": (_I, [_P, _P, _I, _I]),
+    "qvla_layer_scale_groups": (_I, [_P, _P, _P]),
+    "qvla_rotated_absmax_groups": (_I, [_P, _I, _I, _I, _I, _P, _P]),
     "qvla_layer_info": (_I, [_P, _P, _P, _P, _P]),
     "qvla_rotate_quantize": (_I, [_P, _P, _I, _I, _P, _P, _P, _P]),
     "qvla_rotate_quantize_rows": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
@@ -176,6 +179,24 @@ def qvla_layer_destroy(layer: Layer) -> None:
 def qvla_set_step_scales(layer: Layer, scales: np.ndarray) -> None:
     scales = np.ascontiguousarray(scales, dtype=np.float32)
     _check(_lib.qvla_set_step_scales(layer.handle, _ptr(scales), int(scales.shape[0])))
+
+
+def qvla_set_step_group_scales(layer: Layer, scales: np.ndarray) -> None:
+    """Per-step, per-group table [T, G] (float32)."""
+    arr = np.ascontiguousarray(scales, dtype=np.float32)
+    if arr.ndim != 2:
+        raise ValueError("scales must be [T, G]")
+    _check(_lib.qvla_set_step_group_scales(layer.handle, _ptr(arr), arr.shape[0], arr.shape[1]))
+
+
+def qvla_layer_scale_groups(layer: Layer):
+    g, size = ctypes.c_int(), ctypes.c_int()
+    _check(_lib.qvla_layer_scale_groups(layer.handle, ctypes.byref(g), ctypes.byref(size)))
+    return g.value, size.value
+
+
+def qvla_rotated_absmax_groups(x, xdt: int, M: int, K: int, had_block: int, absmax, stream=None) -> None:
+    _check(_lib.qvla_rotated_absmax_groups(_ptr(x), xdt, M, K, had_block, _ptr(absmax), _stream(stream)))
 
 
 def qvla_layer_info(layer: Layer):
