@@ -21,7 +21,8 @@ The line also carries the two layer stacks (skipped with --no-stacks):
   "backbone": 18 layers of hidden 2048 with the gated 16384 MLP, per-token scales, one forward
          pass at M = 816 (TOPS) and at M = 1 (HBM-bound: GB/s of packed weights);
   "dit"."w4a8" and "w4a8_gate_up": the W4A8 variant (8-bit activation codes) on the DiT stack
-         and on the backbone's gate/up projection.
+         and on the backbone's gate/up projection;
+  "dit"."grouped": the DiT stack with Hadamard blocks of 64 and per-step, per-group tables.
 """
 
 from __future__ import annotations
@@ -347,14 +348,15 @@ def _time_replays(fn, reps, flush=None, stream=None):
     return sum(a.elapsed_time(b) for a, b in evs) / reps
 
 
-def _dit_stack(S, Q, W, weights, peaks, act_bits, dev, stream, flush, peak_gbs, peak_src):
+def _dit_stack(S, Q, W, weights, peaks, act_bits, dev, stream, flush, peak_gbs, peak_src, profile=False):
     """One DiT stack (18 blocks, M = 50, T = 10) with int4 or 8-bit activation codes: per-step
-    microseconds with L2 flushed, per rollout, and back to back."""
+    microseconds with L2 flushed, per rollout, and back to back.  peaks[layer] is [T] (one scale
+    per step) or [T, G] (per-group scales)."""
     qmax = np.float32(7 if act_bits == 4 else 127)
     st = S.LinearStack(weights, DIT_M, "f16", "f16", dev, input_sets=DIT_T, act_bits=act_bits)
     for i, w in enumerate(weights):
         for t in range(DIT_T):
-            st.set_input(i, torch.from_numpy(W.dit_layer_input(DIT_SEED, i, t, DIT_M, w.k, DIT_T)), t)
+            st.set_input(i, torch.from_numpy(W.dit_layer_input(DIT_SEED, i, t, DIT_M, w.k, DIT_T, profile)), t)
     st.set_step_tables([p / qmax for p in peaks])
     graphs = [st.capture(t) for t in range(DIT_T)]
     for _ in range(3):
@@ -442,8 +444,23 @@ def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
         peaks.append(np.asarray(row, dtype=np.float32))
     dit = _dit_stack(S, Q, W, weights, peaks, 4, dev, stream, flush, peak_gbs, peak_src)
     dit["w4a8"] = _dit_stack(S, Q, W, weights, peaks, 8, dev, stream, flush, peak_gbs, peak_src)
+    # the paper's rotation configuration: Hadamard blocks of 64, per-step tables per 128-channel
+    # group, inputs with uneven channel magnitudes
+    wb = W.dit_stack_blocks(weights, 64)
+    gpeaks = []
+    for i, w in enumerate(wb):
+        row = []
+        for t in range(DIT_T):
+            xc = torch.from_numpy(W.dit_layer_input(DIT_SEED + 1000, i, t, DIT_CAL_ROWS, w.k, DIT_T, True)).to(
+                dev, torch.float16)
+            gp = torch.zeros(w.k // 128, dtype=torch.float32, device=dev)
+            Q.qvla_rotated_absmax_groups(xc, Q.F16, DIT_CAL_ROWS, w.k, w.had_block, gp, stream)
+            row.append(gp.cpu().numpy())
+        gpeaks.append(np.asarray(row, dtype=np.float32))
+    dit["grouped"] = _dit_stack(S, Q, W, wb, gpeaks, 4, dev, stream, flush, peak_gbs, peak_src, profile=True)
     dit["tables"] = ("per-step, per-layer, calibrated with qvla_rotated_absmax on a separate 16-token draw "
-                     "(absmax / 7; absmax / 127 for the W4A8 variant)")
+                     "(absmax / 7; absmax / 127 for the W4A8 variant); 'grouped': Hadamard blocks of 64 and "
+                     "per-step tables per 128-channel group (qvla_rotated_absmax_groups)")
     w4a8_gu = _w4a8_gate_up(Q, W, dev, stream, flush, peak_tflops)
 
     # ---- backbone forward at M = 816 and M = 1 (per-token scales) ----

@@ -61,9 +61,13 @@ class LinearStack:
         self.ops = sum(2 * m * w.k * (2 * w.n if w.gated else w.n) for w in weights)
 
     def set_step_tables(self, tables) -> None:
-        """One per-step scale table (float32 [T]) per layer."""
+        """One per-step scale table per layer: float32 [T], or [T, G] for per-group scales."""
         for layer, t in zip(self.layers, tables):
-            Q.qvla_set_step_scales(layer, np.asarray(t, dtype=np.float32))
+            t = np.asarray(t, dtype=np.float32)
+            if t.ndim == 2:
+                Q.qvla_set_step_group_scales(layer, t)
+            else:
+                Q.qvla_set_step_scales(layer, t)
 
     @property
     def x(self):

@@ -18,7 +18,7 @@ gives the same tensors on every machine.
 
 from __future__ import annotations
 
-from dataclasses import dataclass, field
+from dataclasses import dataclass, replace, field
 
 import numpy as np
 import torch
@@ -240,12 +240,25 @@ def dit_stack(seed: int = 2, layers: int = 18) -> list:
     return out
 
 
-def dit_layer_input(seed: int, index: int, t: int, m: int, k: int, steps: int = 10) -> np.ndarray:
+def dit_layer_input(seed: int, index: int, t: int, m: int, k: int, steps: int = 10,
+                    channel_profile: bool = False) -> np.ndarray:
     """Input of linear `index` of the DiT stack at denoising step t: N(0, sigma_t^2) [m, k]
     float32 with sigma_t drifting from 4.0 (t = 0) to 0.5 (t = T-1).  Each (index, t) has its
-    own stream, so any subset can be drawn."""
+    own stream, so any subset can be drawn.  channel_profile: every block of 64 channels is
+    also multiplied by its own log-normal factor (spread 0.8, fixed per linear), the uneven
+    channel magnitudes that per-group scales are for."""
     rng = np.random.default_rng([seed, index, t])
-    return rng.standard_normal((m, k), dtype=np.float32) * np.float32(dit_input_std(t, steps))
+    x = rng.standard_normal((m, k), dtype=np.float32) * np.float32(dit_input_std(t, steps))
+    if channel_profile:
+        prof = np.exp(np.random.default_rng([seed, index, 7919]).normal(0.0, 0.8, k // 64)).astype(np.float32)
+        x *= np.repeat(prof, 64)[None, :]
+    return x
+
+
+def dit_stack_blocks(weights, had_block: int = 64) -> list:
+    """The same DiT weights with the paper's rotation block (Sec. 5.1: block size 64) as the
+    layers' Hadamard block, for per-group step scales over 128-channel groups."""
+    return [replace(w, had_block=had_block) for w in weights]
 
 
 BACKBONE_STACK_LAYERS = (("qkv", 2048, 2560, False), ("o", 2048, 2048, False), ("gate_up", 2048, 16384, True),

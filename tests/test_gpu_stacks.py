@@ -88,6 +88,34 @@ def test_dit_stack_w4a8_every_linear():
         st.close()
 
 
+def test_dit_stack_grouped_scales_every_linear():
+    """The DiT stack in the paper's rotation configuration (Hadamard blocks of 64) with
+    per-step, per-group tables over 128-channel groups, calibrated by the oracle on a separate
+    16-token draw of channel-profiled inputs; every linear checked at the first and last step."""
+    weights = W.dit_stack_blocks(W.dit_stack(DIT_SEED), 64)
+    tables = [O.calibrate_step_table_grouped([W.dit_layer_input(DIT_SEED + 1000, i, t, CAL_ROWS, w.k, DIT_T, True)
+                                              for t in range(DIT_T)], w.had_block)
+              for i, w in enumerate(weights)]
+    st = S.LinearStack(weights, DIT_M, "f16", "f16", G.DEV)
+    st.set_step_tables(tables)
+    try:
+        for t in (0, DIT_T - 1):
+            for i, w in enumerate(weights):
+                st.set_input(i, torch.from_numpy(W.dit_layer_input(DIT_SEED, i, t, DIT_M, w.k, DIT_T, True)))
+            g = st.capture(t)
+            for y in st.y:
+                y.fill_(float("nan"))
+            g.replay()
+            torch.cuda.synchronize()
+            G.Q.qvla_check_device(G.stream())
+            for i, w in enumerate(weights):
+                ref = O.grouped_linear(st.x[i].double().cpu().numpy(), w.codes, w.wscale, w.had_block, tables[i], t,
+                                       bias=w.bias, out_fmt="f16")
+                G.assert_output_close(st.y[i].double().cpu().numpy(), ref["y"], "f16")
+    finally:
+        st.close()
+
+
 def _backbone_check(weights, st, rows, seed):
     """Sampled rows of every linear; all output channels of qkv and o, 256 of down, 128 hidden
     units (gate and up rows) of the gated layer.  The oracle unpacks the sampled weight rows."""
