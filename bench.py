@@ -267,20 +267,43 @@ def run_ours(args):
     value = job_value(world, OPS_STEP, K, ms)
 
     # ---- end to end through the public API with host buffers ----
+    # Each step copies its input from pinned host memory, runs both linears through
+    # qvla_w4a4_linear and reads its output back to pinned host memory.  The copies run on their
+    # own streams so that step i + 1's input upload and step i - 1's read-back overlap step i's
+    # kernels (the rotating sets keep the buffers of steps in flight apart): the pipelining a
+    # serving loop does.  The timed region spans the first upload to the last read-back.
     x_host = mlp.x.pin_memory()
     y_host = torch.empty(M, K_IN, dtype=torch.bfloat16).pin_memory()
     K2 = max(1, min(K, 2000))
+    h2d, d2h = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    nset = args.sets
+    in_ready = [torch.cuda.Event() for _ in range(K2)]
+    x_free = [torch.cuda.Event() for _ in range(K2)]   # the set's input has been read
+    y_ready = [torch.cuda.Event() for _ in range(K2)]
+    y_free = [torch.cuda.Event() for _ in range(K2)]   # the set's output has been read back
     barrier(world)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
+    e0.record(h2d)
     for i in range(K2):
-        s = sets[i % args.sets]
-        s["x"].copy_(x_host, non_blocking=True)
+        s = sets[i % nset]
+        with torch.cuda.stream(h2d):
+            if i >= nset:
+                h2d.wait_event(x_free[i - nset])
+            s["x"].copy_(x_host, non_blocking=True)
+            in_ready[i].record(h2d)
+        stream.wait_event(in_ready[i])
+        if i >= nset:
+            stream.wait_event(y_free[i - nset])
         Q.qvla_w4a4_linear(s["gu"], s["x"], M, -1, s["h"], s["ws_gu"], s["ws_gu"].numel(), stream)
+        x_free[i].record(stream)
         Q.qvla_w4a4_linear(s["dn"], s["h"], M, -1, s["y"], s["ws_dn"], s["ws_dn"].numel(), stream)
-        y_host.copy_(s["y"], non_blocking=True)
-    e1.record(stream)
+        y_ready[i].record(stream)
+        with torch.cuda.stream(d2h):
+            d2h.wait_event(y_ready[i])
+            y_host.copy_(s["y"], non_blocking=True)
+            y_free[i].record(d2h)
+    e1.record(d2h)
     torch.cuda.synchronize()
     barrier(world)
     Q.qvla_check_device(stream)
@@ -307,7 +330,9 @@ def run_ours(args):
             "kernels_us": {"rotate_quantize_x": round(rqx_ms * 1e3, 2), "gemm_gate_up": round(gemm_gu_ms * 1e3, 2),
                            "rotate_quantize_h": round(rqh_ms * 1e3, 2), "gemm_down": round(gemm_dn_ms * 1e3, 2)},
             "e2e": {"value": round(e2e, 2), "unit": "TOPS", "h2d_bytes_per_step": M * K_IN * 2,
-                    "d2h_bytes_per_step": M * K_IN * 2, "steps": K2},
+                    "d2h_bytes_per_step": M * K_IN * 2, "steps": K2,
+                    "note": "qvla_w4a4_linear with pinned host input and output copies every step, the copies "
+                            "on their own streams overlapping the neighbouring steps' kernels"},
             "gpu_launches": 4 * K,
             "clocks": clk,
             "cpu_baseline": cpu,

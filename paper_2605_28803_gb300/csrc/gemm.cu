@@ -23,8 +23,10 @@
 // weight rows); for M <= 128 ("swap") it is the weights (128 weight rows x Mpad tokens),
 // so that a small batch does not waste the 128-row MMA.  A small batch has few tiles, so in
 // the weight-major orientation a cluster of up to 8 CTAs shares each tile, splitting K: every
-// CTA leaves its FP32 partial (exact, like the whole sum) in its own shared memory and, after
-// a cluster barrier, sums one slice of the tile's rows over the cluster and applies the epilogue.
+// CTA computes an FP32 partial (exact, like the whole sum) and pushes each slice of its rows,
+// with asynchronous stores that complete on the receiver's mbarrier, to the CTA owning those
+// rows, which sums the slices in its own shared memory and applies the epilogue.  No CTA reads
+// another's shared memory, so the cluster needs no barrier around the reduction.
 //
 // Both kernels of the linear are launched with programmatic stream serialization, so each may
 // start (allocate TMEM, initialise barriers, request weights) while the previous kernel of the
@@ -63,7 +65,9 @@ constexpr uint32_t kEpiBarrier = 1;  // named barrier of the epilogue warps
 // the converters); otherwise it arrives as operand bytes straight from a swizzled TMA load.
 // kPlanes: operand-byte planes per k-block of the activations (2 for 8-bit codes: the high and
 // the low nibbles, each one 128-byte tile against the same weight tile).
-template <int kBN, bool kStageA = true, bool kStageB = true, int kPlanes = 1>
+// kRecv: bytes after the rings where the weight-major split-K reduction receives the partials
+// of the cluster's CTAs.
+template <int kBN, bool kStageA = true, bool kStageB = true, int kPlanes = 1, int kRecv = 0>
 struct Cfg {
   static constexpr int kTileA1 = kBM * kBK;   // bytes of E4M3 of one plane
   static constexpr int kTileB1 = kBN * kBK;
@@ -73,9 +77,10 @@ struct Cfg {
   static constexpr int kRawA = kStageA ? kBM * kBK / 2 : 0;  // packed k-block (64-byte rows)
   static constexpr int kRawB = kStageB ? kBN * kBK / 2 : 0;
   static constexpr int kRaw = kRawA + kRawB;
-  static constexpr int kStagesRaw = (216 * 1024) / (kStage + kRaw);
+  static constexpr int kStagesRaw = (216 * 1024 - kRecv) / (kStage + kRaw);
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
-  static constexpr int kSmem = kStages * (kStage + kRaw) + 1024;  // + alignment slack
+  static constexpr int kRecvOff = kStages * (kStage + kRaw);
+  static constexpr int kSmem = kRecvOff + kRecv + 1024;  // + alignment slack
   static constexpr uint32_t kTmemCols = (2 * kBN) <= 32 ? 32 : (2 * kBN) <= 64 ? 64 : (2 * kBN) <= 128 ? 128 : (2 * kBN) <= 256 ? 256 : 512;
   static_assert(kStages >= 2, "stages");
   static_assert(kRaw % 1024 == 0 && kStage % 1024 == 0, "1024-byte aligned stages");
@@ -217,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   constexpr int kPlanes = kX == 2 ? 2 : 1;
   constexpr bool kStageA = !(kXBytes && !kSwap);  // operand A is the activations unless swapped
   constexpr bool kStageB = !(kXBytes && kSwap);
-  using C = Cfg<kBN, kStageA, kStageB, kPlanes>;
+  using C = Cfg<kBN, kStageA, kStageB, kPlanes, kSwap ? kBM * kBN * 4 : 0>;
   static_assert(kSwap || kBN % 128 == 0, "a weight tile is whole 128-row chunks");
   static_assert(!kGroup || (kBN <= 128 && !kGated && kX == 1), "grouped scales: int4 operand bytes, BN <= 128");
   // TMEM columns: two accumulators, plus the running sum of the grouped mode
@@ -232,6 +237,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   __shared__ __align__(8) uint64_t bar_tfull[2];
   __shared__ __align__(8) uint64_t bar_tempty[2];
   __shared__ __align__(8) uint64_t bar_done;
+  __shared__ __align__(8) uint64_t bar_recv;  // split-K: every CTA's slice of this CTA's rows has landed
   __shared__ uint32_t s_tmem_base;
   __shared__ int s_epi_abort;  // set by an epilogue thread whose wait timed out
   // per-column parameters of the current tile (non-swap): weight scale, code correction, bias
@@ -273,6 +279,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       mbar_init(smem_u32(&bar_tempty[i]), kEpiThreads);
     }
     mbar_init(smem_u32(&bar_done), 1);
+    mbar_init(smem_u32(&bar_recv), 1);
     mbar_init_fence();
     s_epi_abort = 0;
   }
@@ -281,6 +288,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = s_tmem_base;
+  if (kSwap && splits > 1) {
+    // split-K: this CTA receives one slice of its rows from every CTA of the cluster; the
+    // cluster barrier completed before the first send guarantees every receiver's barrier exists
+    if (threadIdx.x == 0) mbar_arrive_expect_tx(smem_u32(&bar_recv), static_cast<uint32_t>(kBM * kBN * 4));
+    cluster_arrive_relaxed();
+  }
   if (threadIdx.x == 0) griddep_launch_dependents();
 
   if (warp == kTmaWarp) {
@@ -756,20 +769,34 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   __syncthreads();
   if constexpr (kSwap) {
     if (splits > 1) {
-      // split-K: every CTA's partial is in its shared memory; CTA r sums rows
-      // [r R, (r + 1) R) of the tile (R = 128 / splits) over the cluster and applies the
-      // epilogue.  All threads take part; an element is 4 consecutive weight rows of one token
-      // column, and its epilogue parameters are fetched one element ahead (the first while the
-      // cluster barrier completes).
-      cluster_arrive();  // this CTA's partial is published
-      const int R4 = kBM / splits / 4;
+      // split-K: every CTA's partial [kBN columns][128 rows] is in its shared memory.  CTA r
+      // owns rows [r R, (r + 1) R) of the tile (R = 128 / splits): each CTA pushes its slice of
+      // those rows into CTA r's receive area ([source CTA][column][R rows]) with asynchronous
+      // stores that complete on CTA r's barrier; CTA r then sums the slices from its own shared
+      // memory and applies the epilogue.  An element is 4 consecutive weight rows of one token
+      // column; its epilogue parameters are fetched one element ahead (the first while the
+      // partials are in flight).  No CTA reads another's shared memory, so none waits for the
+      // others before leaving.
+      cluster_wait();  // pairs with the arrive after set-up: every receive barrier is initialised
+      const int R = kBM / splits;
+      const float* part = reinterpret_cast<const float*>(smem);
+      const uint32_t recv0 = smem_u32(smem + C::kRecvOff);
+      for (int v = threadIdx.x; v < kBN * (kBM / 4); v += kThreads) {
+        const int col = v / (kBM / 4), row = (v % (kBM / 4)) * 4;
+        const int owner = row / R;
+        const float4 val = *reinterpret_cast<const float4*>(part + col * kBM + row);
+        const uint32_t dst = recv0 + static_cast<uint32_t>(((static_cast<int>(krank) * kBN + col) * R + (row - owner * R)) * 4);
+        st_async_v4(mapa_shared(dst, static_cast<uint32_t>(owner)), val,
+                    mapa_shared(smem_u32(&bar_recv), static_cast<uint32_t>(owner)));
+      }
+      const int R4 = R / 4;
       const int unit0 = static_cast<int>(QVLA_UNIT0);
       const int total = unit0 < ntiles && !s_epi_abort ? R4 * kBN : 0;
       const int ta = unit0 % tiles_a, tb = unit0 / tiles_a;
       auto coords = [&](int e, int& n, int& m, int& row, int& col) {
-        row = (static_cast<int>(krank) * R4 + e % R4) * 4;
+        row = (e % R4) * 4;  // within this CTA's R rows
         col = e / R4;
-        n = ta * kBM + row;
+        n = ta * kBM + static_cast<int>(krank) * R + row;
         m = tb * kBN + col;
       };
       griddep_wait();
@@ -780,9 +807,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
         coords(e, n, m, row, col);
         nxt.template load<kGroup>(p, n, m);
       }
-      cluster_wait();
-      const uint32_t part0 = smem_u32(smem);
-      for (; e < total; e += kThreads) {
+      // acquire at cluster scope: the asynchronous stores release their bytes at cluster scope
+      const bool landed = mbar_wait_cluster(smem_u32(&bar_recv), 0);
+      const float* recv = reinterpret_cast<const float*>(smem + C::kRecvOff);
+      for (; landed && e < total; e += kThreads) {
         int n, m, row, col;
         coords(e, n, m, row, col);
         const SplitParams cur = nxt;
@@ -791,20 +819,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
           coords(e + kThreads, n2, m2, r2, c2);
           nxt.template load<kGroup>(p, n2, m2);
         }
-        const uint32_t off = static_cast<uint32_t>((col * kBM + row) * 4);
-        float4 v[8];
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          if (q < splits) v[q] = ld_dsmem_v4(mapa_shared(part0 + off, static_cast<uint32_t>(q)));
         // exact: the partials add up to the tile's accumulator, an integer below 2^24 times 2^-18
-        float4 sum = v[0];
+        float4 sum = *reinterpret_cast<const float4*>(recv + col * R + row);
 #pragma unroll
         for (int q = 1; q < 8; ++q)
           if (q < splits) {
-            sum.x += v[q].x;
-            sum.y += v[q].y;
-            sum.z += v[q].z;
-            sum.w += v[q].w;
+            const float4 v = *reinterpret_cast<const float4*>(recv + (q * kBN + col) * R + row);
+            sum.x += v.x;
+            sum.y += v.y;
+            sum.z += v.z;
+            sum.w += v.w;
           }
         if (kGroup && n < p.N && m < p.M) {  // grouped: the partials are scaled and corrected sums
           const uint32_t lo = pack2<OutT>(fmaf(sum.x, cur.ws.x, cur.bs.x), fmaf(sum.y, cur.ws.y, cur.bs.y));
@@ -827,7 +851,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
                           static_cast<int32_t>(a3));
         }
       }
-      cluster_sync();  // no CTA leaves while another still reads its partial
     }
   }
   tc_fence_after();
@@ -919,7 +942,7 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   constexpr int kPlanes = kX == 2 ? 2 : 1;
   constexpr bool kStageA = !(kXBytes && !kSwap);
   constexpr bool kStageB = !(kXBytes && kSwap);
-  using C = Cfg<kBN, kStageA, kStageB, kPlanes>;
+  using C = Cfg<kBN, kStageA, kStageB, kPlanes, kSwap ? kBM * kBN * 4 : 0>;
   Params p;
   if (kSwap) {
     p.a = a.wq;
