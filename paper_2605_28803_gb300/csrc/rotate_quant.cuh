@@ -191,7 +191,7 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
 #pragma unroll
     for (int i = 0; i < kN; ++i) v[i] = make_float2(0.0f, 0.0f);
   }
-  __syncthreads();
+  __syncthreads();  // the reduction slots are cleared before any thread adds to them
 
   constexpr int kLowBits = kLogB < kP ? kLogB : kP;
   fwht_regs<kN, 0, kLowBits>(v);
@@ -203,7 +203,10 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
       const int line = j;
       s4[line * kNV + (c ^ (line & (kNV - 1)))] = make_float4(v[2 * c].x, v[2 * c].y, v[2 * c + 1].x, v[2 * c + 1].y);
     }
-    __syncthreads();
+    // A Hadamard block's 2^kR threads (at most 32, starting at a multiple of 2^kR) lie in one
+    // warp, and each reads back only its block's lines: the warp alone must have stored them.
+    static_assert(kR <= 5, "a Hadamard block's threads fit in one warp");
+    __syncwarp();
     const int jlo = j & ((1 << kR) - 1);
     const int jhi = j >> kR;
 #pragma unroll
