@@ -781,13 +781,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       const int R = kBM / splits;
       const float* part = reinterpret_cast<const float*>(smem);
       const uint32_t recv0 = smem_u32(smem + C::kRecvOff);
-      for (int v = threadIdx.x; v < kBN * (kBM / 4); v += kThreads) {
-        const int col = v / (kBM / 4), row = (v % (kBM / 4)) * 4;
+      // kThreads is a multiple of kBM / 4, so a thread's row (and owner) is the same at every step
+      static_assert(kThreads % (kBM / 4) == 0, "fixed row per thread");
+      {
+        const int row = (static_cast<int>(threadIdx.x) % (kBM / 4)) * 4;
         const int owner = row / R;
-        const float4 val = *reinterpret_cast<const float4*>(part + col * kBM + row);
-        const uint32_t dst = recv0 + static_cast<uint32_t>(((static_cast<int>(krank) * kBN + col) * R + (row - owner * R)) * 4);
-        st_async_v4(mapa_shared(dst, static_cast<uint32_t>(owner)), val,
-                    mapa_shared(smem_u32(&bar_recv), static_cast<uint32_t>(owner)));
+        const uint32_t rbar = mapa_shared(smem_u32(&bar_recv), static_cast<uint32_t>(owner));
+        const uint32_t rdst = mapa_shared(recv0, static_cast<uint32_t>(owner)) +
+                              static_cast<uint32_t>((static_cast<int>(krank) * kBN * R + (row - owner * R)) * 4);
+        for (int col = static_cast<int>(threadIdx.x) / (kBM / 4); col < kBN; col += kThreads / (kBM / 4))
+          st_async_v4(rdst + static_cast<uint32_t>(col * R * 4), *reinterpret_cast<const float4*>(part + col * kBM + row), rbar);
       }
       const int R4 = R / 4;
       const int unit0 = static_cast<int>(QVLA_UNIT0);
