@@ -406,12 +406,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
         for (int i = 0; i < kPer; ++i)
           if (kChunks % kConvThreads == 0 || ct + i * kConvThreads < kChunks)
             v[i] = *reinterpret_cast<const uint4*>(src + 16 * (ct + i * kConvThreads));
-        mbar_arrive(smem_u32(&bar_raw_empty[s]));  // the staged k-block is in registers now
 #pragma unroll
         for (int i = 0; i < kPer; ++i)
           if (kChunks % kConvThreads == 0 || ct + i * kConvThreads < kChunks)
             store_chunk(dst + d_row[i], d_o0[i], d_o1[i], v[i]);
+        // The staged k-block is released only now: the conversions above consumed every loaded
+        // value, so the loads have completed, and the proxy fence orders them (and the stores)
+        // before the async proxy's next accesses, the TMA's refill of the staging stage and the
+        // MMAs' reads of the expanded one.  Releasing it straight after issuing the loads let
+        // a refill overwrite the stage under loads still in flight (measured: the MMA of k-block
+        // j then used some rows of k-block j + kStages).
         fence_proxy_async_smem();
+        mbar_arrive(smem_u32(&bar_raw_empty[s]));
         mbar_arrive(smem_u32(&bar_full[s]));
       }
     }

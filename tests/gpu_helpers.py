@@ -15,7 +15,7 @@ def stream():
 
 
 def rotate_quantize_rows(x: torch.Tensor, had: int, step_scale=None):
-    """GPU rotate + quantise of an [M, K] tensor; returns (codes int8 [M,K], scale f32 [M], sum int [M])."""
+    """GPU rotate + quantise of an [M, K] tensor; returns (packed codes uint8 [M, K/2], scale f32 [M], sum int [M])."""
     M, K = x.shape
     xdt = {torch.float16: Q.F16, torch.bfloat16: Q.BF16, torch.float32: Q.F32}[x.dtype]
     xg = x.to(DEV).contiguous()

@@ -10,6 +10,7 @@ import numpy as np
 import pytest
 
 from oracle import qvla_oracle as O
+from paper_2605_28803_gb300 import qvla as Q
 from tests import gpu_helpers as G
 
 pytestmark = pytest.mark.gpu
@@ -41,6 +42,9 @@ def _run(M, N, K, seed, ydt="f16", with_bias=True):
     # weight-major split-K: a cluster of 2 with several reduction elements per thread, 5
     # k-blocks over 4 CTAs (uneven slices) with a ragged weight tile, a decode row at K = 16384
     (100, 8192, 1024), (33, 400, 640), (1, 2048, 16384),
+    # token-major at larger M: 128- and 256-wide tiles with ragged last token tiles (1100, 1450)
+    # beside a ragged weight tile, and several tiles per persistent CTA (640 x 16384)
+    (1024, 384, 1024), (1100, 1008, 512), (1450, 2048, 1024), (2048, 4096, 256), (640, 16384, 2048),
 ])
 def test_gemm_accumulator_bit_exact(M, N, K):
     acc, ref_acc, y, ref_y = _run(M, N, K, seed=M * 7 + N + K)
@@ -90,3 +94,23 @@ def test_gemm_zero_scale_gives_bias():
     y, _ = G.gemm(layer, O.pack_int4(qx), np.zeros(M, np.float32), qx.astype(np.int64).sum(1))
     layer.close()
     assert np.array_equal(y, np.broadcast_to(O.round_to_format(bias.astype(np.float64), "f16"), (M, N)))
+
+
+@pytest.mark.parametrize("M,H,K", [(512, 128, 256), (600, 256, 512), (1450, 384, 1024)])
+def test_gated_gemm_bit_exact(M, H, K):
+    """Gated layers (gate and up rows of a hidden unit in one 256-wide tile): [gate | up]
+    accumulators bit-exact and h = gelu(gate) * up within the output tolerance, with ragged
+    last token tiles (600, 1450) and a ragged tile of hidden units (H = 384)."""
+    rng = np.random.default_rng(M + H + K)
+    qx = _codes(rng, M, K, -7, 7)
+    qg, qu = _codes(rng, H, K), _codes(rng, H, K)
+    dx = rng.uniform(0.01, 0.3, M).astype(np.float32)
+    dg, du = (rng.uniform(0.001, 0.02, H).astype(np.float32) for _ in range(2))
+    layer = Q.qvla_layer_create_gated(H, K, 1, Q.F16, Q.BF16, O.pack_int4(qg), dg, O.pack_int4(qu), du)
+    y, acc = G.gemm(layer, O.pack_int4(qx), dx, qx.astype(np.int64).sum(1), ydt="bf16")
+    layer.close()
+    ag, au = O.int_gemm(qx, qg), O.int_gemm(qx, qu)
+    assert np.array_equal(acc, np.concatenate([ag, au], axis=1))
+    gate = O.dequant_output(ag, dx, dg, None, "bf16")
+    up = O.dequant_output(au, dx, du, None, "bf16")
+    G.assert_output_close(y, O.round_to_format(O.gated_glue(gate, up), "bf16"), "bf16")
