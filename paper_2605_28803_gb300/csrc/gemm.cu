@@ -215,18 +215,26 @@ struct SplitParams {
 // kGroup: per-step, per-group activation scales.  Each group's k-blocks accumulate into a fresh
 // TMEM buffer; the epilogue removes that group's zero point exactly, scales by the group's
 // Delta and adds the result into a running FP32 sum held in TMEM beside the two buffers.
-template <int kBN, bool kSwap, bool kGated, int kX, typename OutT, bool kGroup = false>
+// kPair: token-major on a CTA pair (cluster of 2): one 2-SM MMA (cta_group::2, M = 256) per
+// step covers 256 tokens x kBN weight rows; each CTA stages its 128 token rows and half of the
+// weight rows and receives its 128 rows of the accumulator in its own TMEM.  The leader (rank 0)
+// issues the MMAs; the peer's activation tiles complete on the leader's barrier directly, and one
+// peer thread forwards its converters' completion of each stage.
+template <int kBN, bool kSwap, bool kGated, int kX, typename OutT, bool kGroup = false, bool kPair = false>
 __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_constant__ CUtensorMap tmap_a,
                                                                  const __grid_constant__ CUtensorMap tmap_b, Params p) {
   constexpr bool kXBytes = kX >= 1;
   constexpr int kPlanes = kX == 2 ? 2 : 1;
   constexpr bool kStageA = !(kXBytes && !kSwap);  // operand A is the activations unless swapped
   constexpr bool kStageB = !(kXBytes && kSwap);
-  using C = Cfg<kBN, kStageA, kStageB, kPlanes, kSwap ? kBM * kBN * 4 : 0>;
+  static_assert(!kPair || (!kSwap && !kGroup && kX <= 1), "pairs: token-major, int4 activations");
+  constexpr int kBS = kPair ? kBN / 2 : kBN;  // weight rows this CTA stages
+  using C = Cfg<kBS, kStageA, kStageB, kPlanes, kSwap ? kBM * kBN * 4 : 0>;
   static_assert(kSwap || kBN % 128 == 0, "a weight tile is whole 128-row chunks");
   static_assert(!kGroup || (kBN <= 128 && !kGated && kX == 1), "grouped scales: int4 operand bytes, BN <= 128");
   // TMEM columns: two accumulators, plus the running sum of the grouped mode
-  constexpr uint32_t kTmemCols = !kGroup ? C::kTmemCols : (3 * kBN <= 64 ? 64 : 3 * kBN <= 128 ? 128 : 3 * kBN <= 256 ? 256 : 512);
+  constexpr uint32_t kTmemCols = kPair ? (2 * kBN <= 256 ? 256 : 512)
+                                       : !kGroup ? C::kTmemCols : (3 * kBN <= 64 ? 64 : 3 * kBN <= 128 ? 128 : 3 * kBN <= 256 ? 256 : 512);
   extern __shared__ uint8_t dyn_smem[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~uintptr_t(1023));
 
@@ -248,7 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  const int tiles_a = (p.rows_a + kBM - 1) / kBM;
+  const int tiles_a = (p.rows_a + (kPair ? 2 : 1) * kBM - 1) / ((kPair ? 2 : 1) * kBM);
   const int tiles_b = (p.rows_b + kBN - 1) / kBN;
   const int ntiles = tiles_a * tiles_b;
   const int nkb_all = p.K / kBK;
@@ -256,6 +264,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   // taking k-blocks [kb0, kb1); without a split every CTA runs whole tiles persistently
   const int splits = kSwap ? p.splits : 1;
   const uint32_t krank = (kSwap && splits > 1) ? cluster_ctarank() : 0u;
+  const uint32_t prank = kPair ? cluster_ctarank() : 0u;  // 0: the pair's leader, which issues the MMAs
+  const int udiv = kPair ? 2 : splits;                      // CTAs per work unit
   // (grouped scales: the split falls on group boundaries, so each group's partial is whole)
   const int kb0 = kGroup ? ((p.ngroups * static_cast<int>(krank)) / splits) * p.gkb
                          : (nkb_all * static_cast<int>(krank)) / splits;
@@ -263,29 +273,39 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
                          : (nkb_all * (static_cast<int>(krank) + 1)) / splits;
   // this CTA's first tile and the tile stride, read where they are used (held in registers
   // across the role loops they would cost a register in every role)
-#define QVLA_UNIT0 (blockIdx.x / static_cast<unsigned>(splits))
-#define QVLA_NUNITS (gridDim.x / static_cast<unsigned>(splits))
+#define QVLA_UNIT0 (blockIdx.x / static_cast<unsigned>(udiv))
+#define QVLA_NUNITS (gridDim.x / static_cast<unsigned>(udiv))
   uint8_t* const raw = smem + C::kStages * C::kStage;  // staging ring after the expanded stages
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(smem_u32(&bar_raw_full[s]), 1);
       mbar_init(smem_u32(&bar_raw_empty[s]), kConvThreads);
-      mbar_init(smem_u32(&bar_full[s]), kConvThreads + (kXBytes ? 1 : 0));  // + the TMA thread's byte count
+      // + the TMA thread's byte count; a pair's leader also counts the peer's forwarder, while the
+      // peer's own barrier counts its converters only
+      mbar_init(smem_u32(&bar_full[s]), kPair && prank != 0 ? kConvThreads
+                                                            : kConvThreads + (kXBytes ? 1 : 0) + (kPair ? 1 : 0));
       mbar_init(smem_u32(&bar_empty[s]), 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&bar_tfull[i]), 1);
-      mbar_init(smem_u32(&bar_tempty[i]), kEpiThreads);
+      mbar_init(smem_u32(&bar_tempty[i]), kEpiThreads + (kPair ? kEpiWarps : 0));
     }
     mbar_init(smem_u32(&bar_done), 1);
     mbar_init(smem_u32(&bar_recv), 1);
     mbar_init_fence();
     s_epi_abort = 0;
   }
-  if (warp == kMmaWarp) tmem_alloc<kTmemCols>(smem_u32(&s_tmem_base));
+  if (warp == kMmaWarp) {
+    if constexpr (kPair) {
+      tmem_alloc_pair<kTmemCols>(smem_u32(&s_tmem_base));
+    } else {
+      tmem_alloc<kTmemCols>(smem_u32(&s_tmem_base));
+    }
+  }
   tc_fence_before();
   __syncthreads();
+  if constexpr (kPair) cluster_sync();  // both CTAs' barriers exist before any arrival crosses the pair
   tc_fence_after();
   const uint32_t tmem_base = s_tmem_base;
   if (kSwap && splits > 1) {
@@ -333,11 +353,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
               if constexpr (kSwap) {
                 bulk_load(dst, p.a + (static_cast<size_t>(ta) * nkb_all + kb) * 8192, 8192, bar);
               } else {
-                tma_load_2d(dst, &tmap_a, kb * (kBK / 2), ta * kBM, bar);
+                tma_load_2d(dst, &tmap_a, kb * (kBK / 2), kPair ? ta * 2 * kBM + static_cast<int>(prank) * kBM : ta * kBM, bar);
               }
             }
             if constexpr (kStageB) {
-              if constexpr (!kSwap) {
+              if constexpr (kPair) {
+                // this CTA's half of the weight tile: chunk 2 tb + rank (kBN 256), or half of chunk tb
+                if constexpr (kBN == 256) {
+                  bulk_load(dst + C::kRawA, p.b + (static_cast<size_t>(tb * 2 + prank) * nkb_all + kb) * 8192, 8192, bar);
+                } else {
+                  bulk_load(dst + C::kRawA, p.b + (static_cast<size_t>(tb) * nkb_all + kb) * 8192 + prank * 4096, 4096, bar);
+                }
+              } else if constexpr (!kSwap) {
 #pragma unroll
                 for (int c = 0; c < kBN / 128; ++c)
                   bulk_load(dst + C::kRawA + c * 8192,
@@ -352,7 +379,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
             if (!mbar_wait(smem_u32(&bar_empty[s]), ph ^ 1u)) { ok = false; break; }
             const uint32_t fb = smem_u32(&bar_full[s]);
             const uint32_t e = smem_u32(smem + s * C::kStage);
-            if constexpr (!kSwap) {
+            if constexpr (kPair) {
+              // both CTAs' activation rows complete on the leader's barrier
+              if (prank == 0) mbar_arrive_expect_tx(fb, 2 * C::kTileA);
+              tma_load_2d_pair(e, &tmap_a, kb * kBK, ta * 2 * kBM + static_cast<int>(prank) * kBM, mapa_shared(fb, 0));
+            } else if constexpr (!kSwap) {
               mbar_arrive_expect_tx(fb, C::kTileA);
 #pragma unroll
               for (int pl = 0; pl < kPlanes; ++pl)
@@ -377,7 +408,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     // ------------------------------------------------------------------ converters
     const int ct = threadIdx.x - (kTmaWarp + 1) * 32;  // 0 .. kConvThreads-1
     constexpr int kChunksA = kStageA ? kBM * 4 : 0;     // 16-byte packed chunks per k-block
-    constexpr int kChunks = kChunksA + (kStageB ? kBN * 4 : 0);
+    constexpr int kChunks = kChunksA + (kStageB ? kBS * 4 : 0);
     constexpr int kPer = (kChunks + kConvThreads - 1) / kConvThreads;
     // destination of each of this thread's chunks: tile byte offset of the row and the two
     // swizzled 16-byte columns; the staged chunk c sits at byte 16 c of the staging k-block
@@ -423,7 +454,47 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0 && kGroup) {
+    if (kPair && lane == 0 && prank == 0) {
+      constexpr uint32_t kIdesc = idesc_e4m3_f32(2 * kBM, kBN);
+      int it = 0, tile_iter = 0;
+      bool ok = true;
+      for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS, ++tile_iter) {
+        const int buf = tile_iter & 1;
+        const uint32_t aph = static_cast<uint32_t>(tile_iter >> 1) & 1u;
+        if (!mbar_wait(smem_u32(&bar_tempty[buf]), aph ^ 1u)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t d = tmem_base + static_cast<uint32_t>(buf * kBN);
+        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+          const int s = it % C::kStages;
+          const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
+          if (!mbar_wait(smem_u32(&bar_full[s]), ph)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + s * C::kStage);
+          const uint32_t sb = sa + C::kTileA;
+#pragma unroll
+          for (int kk = 0; kk < kBK / 32; ++kk)
+            mma_e4m3_pair(d, smem_desc_sw128(sa + kk * 32), smem_desc_sw128(sb + kk * 32), kIdesc,
+                          (kb != kb0 || kk != 0) ? 1u : 0u);
+          mma_commit_pair(smem_u32(&bar_empty[s]), 3);  // both CTAs' stage s is free
+        }
+        if (!ok) break;
+        mma_commit_pair(smem_u32(&bar_tfull[buf]), 3);
+      }
+      mma_commit_pair(smem_u32(&bar_done), 1);
+      mbar_wait(smem_u32(&bar_done), 0);
+    } else if (kPair && lane == 0) {
+      // the peer's forwarder: once this CTA's converters have filled stage s, one arrival tells
+      // the leader (the converters themselves arrive locally)
+      int it = 0;
+      bool ok = true;
+      for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS)
+        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+          const int s = it % C::kStages;
+          if (!mbar_wait(smem_u32(&bar_full[s]), static_cast<uint32_t>(it / C::kStages) & 1u)) { ok = false; break; }
+          mbar_arrive_peer(mapa_shared(smem_u32(&bar_full[s]), 0));
+        }
+    } else if (kPair) {
+    } else if (lane == 0 && kGroup) {
       // one accumulator per scale group, alternating between the two buffers group by group
       constexpr uint32_t kIdesc = idesc_e4m3_f32(kBM, kBN);
       int it = 0, gi = 0;
@@ -624,7 +695,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       }
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(warp * 32) << 16) + static_cast<uint32_t>(buf * kBN);
-      const int ra = ta * kBM + et;  // this thread's MMA-A row
+      const int ra = kPair ? ta * 2 * kBM + static_cast<int>(prank) * kBM + et : ta * kBM + et;  // this thread's MMA-A row
       if constexpr (!kSwap && !kGated) {
         // rows = tokens m, columns = weight rows n
         const int m = ra;
@@ -767,12 +838,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
         }
       }
       tc_fence_before();
-      mbar_arrive(smem_u32(&bar_tempty[buf]));
+      if (kPair && prank != 0) {  // the peer's epilogue warps report to the leader
+        __syncwarp();
+        if (lane == 0) mbar_arrive_peer(mapa_shared(smem_u32(&bar_tempty[buf]), 0));
+      } else {
+        mbar_arrive(smem_u32(&bar_tempty[buf]));
+      }
     }
   }
 
   tc_fence_before();
   __syncthreads();
+  if constexpr (kPair) cluster_sync();  // the leader's MMAs into this CTA's TMEM are complete
   if constexpr (kSwap) {
     if (splits > 1) {
       // split-K: every CTA's partial [kBN columns][128 rows] is in its shared memory.  CTA r
@@ -863,7 +940,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     }
   }
   tc_fence_after();
-  if (warp == kMmaWarp) tmem_dealloc<kTmemCols>(tmem_base);
+  if (warp == kMmaWarp) {
+    if constexpr (kPair) {
+      tmem_dealloc_pair<kTmemCols>(tmem_base);
+    } else {
+      tmem_dealloc<kTmemCols>(tmem_base);
+    }
+  }
 #undef QVLA_UNIT0
 #undef QVLA_NUNITS
 }
@@ -945,13 +1028,13 @@ int max_active_clusters(const void* kern, const cudaLaunchConfig_t& cfg) {
   return n;
 }
 
-template <int kBN, bool kSwap, bool kGated, int kX, typename OutT, bool kGroup = false>
+template <int kBN, bool kSwap, bool kGated, int kX, typename OutT, bool kGroup = false, bool kPair = false>
 cudaError_t launch_cfg(const GemmArgs& a) {
   constexpr bool kXBytes = kX >= 1;
   constexpr int kPlanes = kX == 2 ? 2 : 1;
   constexpr bool kStageA = !(kXBytes && !kSwap);
   constexpr bool kStageB = !(kXBytes && kSwap);
-  using C = Cfg<kBN, kStageA, kStageB, kPlanes, kSwap ? kBM * kBN * 4 : 0>;
+  using C = Cfg<kPair ? kBN / 2 : kBN, kStageA, kStageB, kPlanes, kSwap ? kBM * kBN * 4 : 0>;
   Params p;
   if (kSwap) {
     p.a = a.wq;
@@ -982,9 +1065,10 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   p.M = a.M;
   p.N = a.N;
   p.ldy = a.gated ? a.N / 2 : a.N;
-  const int tiles = ((p.rows_a + kBM - 1) / kBM) * ((p.rows_b + kBN - 1) / kBN);
+  const int tm = kPair ? (p.rows_a + 2 * kBM - 1) / (2 * kBM) : (p.rows_a + kBM - 1) / kBM;
+  const int tiles = tm * ((p.rows_b + kBN - 1) / kBN);
   if (tiles == 0) return cudaSuccess;
-  auto kern = gemm_w4a4_kernel<kBN, kSwap, kGated, kX, OutT, kGroup>;
+  auto kern = gemm_w4a4_kernel<kBN, kSwap, kGated, kX, OutT, kGroup, kPair>;
   cudaError_t e = prepare_kernel(reinterpret_cast<const void*>(kern), C::kSmem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -1013,10 +1097,15 @@ cudaError_t launch_cfg(const GemmArgs& a) {
     }
   }
   p.splits = splits;
-  attr[1].val.clusterDim.x = static_cast<unsigned>(splits);
-  cfg.gridDim = dim3(splits > 1 ? tiles * splits : (tiles < a.num_sms ? tiles : a.num_sms));
+  attr[1].val.clusterDim.x = static_cast<unsigned>(kPair ? 2 : splits);
+  if (kPair) {
+    const int pairs = a.num_sms / 2;
+    cfg.gridDim = dim3(2 * (tiles < pairs ? tiles : pairs));
+  } else {
+    cfg.gridDim = dim3(splits > 1 ? tiles * splits : (tiles < a.num_sms ? tiles : a.num_sms));
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = splits > 1 ? 2 : 1;  // a cluster launch only when K is split
+  cfg.numAttrs = (kPair || splits > 1) ? 2 : 1;  // a cluster launch for pairs and when K is split
   // a tensor map for the activations only (the weights arrive as contiguous chunks)
   CUtensorMap ta = {}, tb = {};
   if constexpr (kSwap) {
@@ -1045,17 +1134,64 @@ cudaError_t launch_grouped(const GemmArgs& a) {
   return launch_cfg<128, true, false, 1, OutT, true>(a);
 }
 
+// Token-major tile shapes and their estimated launch times (ns): a fixed cost plus, per wave of
+// persistent CTAs (or CTA pairs), a per-tile cost and a cost per k-block, fitted to GB300
+// measurements (M 256-8192, K 1024-16384; pairs only from K = 1024): single CTAs with 128- / 256-wide tiles 2300 + waves x
+// (2000 + 344 / k-block) and 2000 + waves x (2500 + 560 / k-block); CTA pairs (256 tokens over two
+// SMs, half the weight rows staged per SM) 3900 + waves x (1000 + 351 / k-block) and 3800 + waves
+// x (2900 + 375 / k-block).  A pair wave holds half as many tiles, each of twice the tokens.
+enum class TileShape { kSingle128, kSingle256, kPair128, kPair256 };
+
+TileShape token_major_shape(const GemmArgs& a) {
+  const long nkb = a.K / kBK, sms = a.num_sms, npairs = a.num_sms / 2;
+  const long t1 = (a.M + kBM - 1) / kBM, t2 = (a.M + 2 * kBM - 1) / (2 * kBM);
+  const long n128 = a.gated ? 0 : (a.N + 127) / 128, n256 = (a.N + 255) / 256;
+  auto est = [nkb](long tiles, long units, long fixed, long per_tile, long per_kb) {
+    return fixed + (tiles + units - 1) / units * (per_tile + nkb * per_kb);
+  };
+  TileShape best = TileShape::kSingle256;
+  long t = est(t1 * n256, sms, 2000, 2500, 560);
+  auto consider = [&](TileShape s, long v) {
+    if (v < t) {
+      t = v;
+      best = s;
+    }
+  };
+  if (n128) consider(TileShape::kSingle128, est(t1 * n128, sms, 2300, 2000, 344));
+  // pairs need a few k-blocks per tile to hide their larger per-tile hand-over (measured at
+  // K = 256: 12% slower than single CTAs where this estimate favoured the pair)
+  if (a.M > kBM && npairs > 0 && nkb >= 8) {
+    consider(TileShape::kPair256, est(t2 * n256, npairs, 3800, 2900, 375));
+    if (n128) consider(TileShape::kPair128, est(t2 * n128, npairs, 3900, 1000, 351));
+  }
+  return best;
+}
+
 template <int kX, typename OutT>
 cudaError_t launch_out(const GemmArgs& a) {
-  if (a.gated) return launch_cfg<256, false, true, kX, OutT>(a);  // gate/up pairs share a 256-row tile
-  if (a.M > 128) {
-    // tile width by estimated time: waves of persistent CTAs x tile width (a narrower tile
-    // wins when the wide one leaves SMs idle, e.g. few output channels and a long K)
-    const long tm = (a.M + kBM - 1) / kBM;
-    const long w256 = (tm * ((a.N + 255) / 256) + a.num_sms - 1) / a.num_sms;
-    const long w128 = (tm * ((a.N + 127) / 128) + a.num_sms - 1) / a.num_sms;
-    if (w128 * 128 < w256 * 256) return launch_cfg<128, false, false, kX, OutT>(a);
-    return launch_cfg<256, false, false, kX, OutT>(a);
+  if (a.gated || a.M > 128) {
+    if constexpr (kX == 2) {
+      // 8-bit activation planes: single CTAs; tile width by waves x tile width
+      if (a.gated) return launch_cfg<256, false, true, kX, OutT>(a);  // gate/up pairs share a 256-row tile
+      const long tm = (a.M + kBM - 1) / kBM;
+      const long w256 = (tm * ((a.N + 255) / 256) + a.num_sms - 1) / a.num_sms;
+      const long w128 = (tm * ((a.N + 127) / 128) + a.num_sms - 1) / a.num_sms;
+      if (w128 * 128 < w256 * 256) return launch_cfg<128, false, false, kX, OutT>(a);
+      return launch_cfg<256, false, false, kX, OutT>(a);
+    } else {
+      // gated layers always take 256-wide tiles: a tile's gate and up rows meet in one epilogue
+      switch (token_major_shape(a)) {
+        case TileShape::kPair256:
+          return a.gated ? launch_cfg<256, false, true, kX, OutT, false, true>(a)
+                         : launch_cfg<256, false, false, kX, OutT, false, true>(a);
+        case TileShape::kPair128:
+          return launch_cfg<128, false, false, kX, OutT, false, true>(a);
+        case TileShape::kSingle128:
+          return launch_cfg<128, false, false, kX, OutT>(a);
+        default:
+          return a.gated ? launch_cfg<256, false, true, kX, OutT>(a) : launch_cfg<256, false, false, kX, OutT>(a);
+      }
+    }
   }
   const int mpad = (a.M + 15) / 16 * 16;
   if (mpad <= 16) return launch_cfg<16, true, false, kX, OutT>(a);

@@ -99,6 +99,14 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, int 
       "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(bar)
       : "memory");
 }
+// The same load for one CTA of a 2-SM pair: the bytes land in this CTA's shared memory and
+// complete on the mbarrier at cluster_bar (from mapa_shared), which may be in either CTA.
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void* tmap, int x, int y, uint32_t cluster_bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2 [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(cluster_bar)
+      : "memory");
+}
 // A contiguous block of global memory into shared memory (both 16-byte aligned, bytes a
 // multiple of 16), completing `bytes` of the mbarrier's transaction count.
 __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
@@ -159,6 +167,13 @@ __device__ __forceinline__ float4 ld_dsmem_v4(uint32_t cluster_addr) {
 // Arrive (release at cluster scope) on an mbarrier of another CTA of the cluster.
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+// Arrive on the other CTA of a 2-SM pair with the default semantics, the form of cluster
+// pipelines whose consumer waits at CTA scope: the waiting thread only issues tensor-core
+// work, whose operands the arriving thread's CTA-scope arrive has already made visible to the
+// async proxy.
+__device__ __forceinline__ void mbar_arrive_peer(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 // Wait on a local mbarrier that other CTAs arrive on (acquire at cluster scope), bounded.
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
