@@ -218,8 +218,9 @@ struct SplitParams {
 // kPair: token-major on a CTA pair (cluster of 2): one 2-SM MMA (cta_group::2, M = 256) per
 // step covers 256 tokens x kBN weight rows; each CTA stages its 128 token rows and half of the
 // weight rows and receives its 128 rows of the accumulator in its own TMEM.  The leader (rank 0)
-// issues the MMAs; the peer's activation tiles complete on the leader's barrier directly, and one
-// peer thread forwards its converters' completion of each stage.
+// issues the MMAs; operand-byte activation tiles of both CTAs complete on the leader's barrier
+// directly, and one peer thread forwards the completion of each stage by the peer's converters
+// (its half of the weight rows, and with packed activations its token rows too).
 template <int kBN, bool kSwap, bool kGated, int kX, typename OutT, bool kGroup = false, bool kPair = false>
 __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_constant__ CUtensorMap tmap_a,
                                                                  const __grid_constant__ CUtensorMap tmap_b, Params p) {
@@ -494,6 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
           mbar_arrive_peer(mapa_shared(smem_u32(&bar_full[s]), 0));
         }
     } else if (kPair) {
+      // the other lanes of a pair's MMA warp have no role
     } else if (lane == 0 && kGroup) {
       // one accumulator per scale group, alternating between the two buffers group by group
       constexpr uint32_t kIdesc = idesc_e4m3_f32(kBM, kBN);
