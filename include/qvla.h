@@ -170,6 +170,27 @@ qvla_status qvla_set_step_scales(qvla_layer* layer, const float* scales, int T);
  * QVLA_ERR_UNSUPPORTED (per-token calls, step == -1, are unaffected).  Synchronous. */
 qvla_status qvla_set_step_group_scales(qvla_layer* layer, const float* scales, int T, int G);
 
+/* Online data-dependent rotation for a layer whose activations cannot take x . P . BlockDiag(U_b)
+ * upstream (Sec. 4.1, Eq. 4-5: layers that share one input but fold different P and U_b, such
+ * as Q, K and V).  With it set, qvla_w4a4_linear, qvla_w4a4_linear_noalloc and
+ * qvla_linear_quantize first form x' = x . P . BlockDiag(U_b) in the workspace -- float32
+ * products summed in the order i = 0 .. rot_block - 1, one rounding to the activation dtype --
+ * and run the Hadamard factor and the quantiser on x'; the workspace grows by M x K elements of
+ * the activation dtype (qvla_linear_workspace_bytes accounts for it).  Pack the weights with the
+ * same perm and rot (qvla_pack_weights_host).  qvla_rotate_quantize and qvla_w4a8_linear refuse
+ * such a layer (QVLA_ERR_UNSUPPORTED).
+ *   perm       host int32 [K] or NULL (identity): column j of x.P is column perm[j] of x.
+ *   rot        host float64 [K/rot_block][rot_block][rot_block], row-major U_b (uploaded as
+ *              float32), or NULL (U = I; perm alone).  Orthogonality is the caller's promise.
+ *   rot_block  16, 32 or 64 (QVLA_ERR_UNSUPPORTED otherwise), dividing K.
+ * perm == NULL and rot == NULL removes the online rotation.  Synchronous. */
+qvla_status qvla_layer_set_online_rotation(qvla_layer* layer, const int32_t* perm, const double* rot, int rot_block);
+
+/* The layer's online rotation alone: out = x . P . BlockDiag(U_b) as above (x, out device
+ * [M][K] of the layer's activation dtype, distinct buffers), e.g. to calibrate step tables on the
+ * values the quantiser sees.  QVLA_ERR_INVALID_ARG if the layer has no online rotation. */
+qvla_status qvla_online_rotate(const qvla_layer* layer, const void* x, int M, void* out, void* stream);
+
 /* The layer's scale groups: G groups of `group` channels (group = max(128, had_block)). */
 qvla_status qvla_layer_scale_groups(const qvla_layer* layer, int* G, int* group);
 
@@ -230,7 +251,8 @@ qvla_status qvla_gemm_w4a4(const qvla_layer* layer, const uint8_t* xq, const flo
 
 /* Bytes of device workspace qvla_w4a4_linear needs for M rows (a multiple of 256): the codes
  * travel between its two kernels as one tensor-core operand byte each (M x K bytes), plus the
- * scales, the code sums and the per-group code sums (M x G x 4 bytes). */
+ * scales, the code sums and the per-group code sums (M x G x 4 bytes), and, for a layer with an
+ * online rotation, x . P . BlockDiag(U_b) (M x K elements of the activation dtype). */
 size_t qvla_linear_workspace_bytes(const qvla_layer* layer, int M);
 
 /* The whole online linear (Sec. 4): rotate + quantise x (as qvla_rotate_quantize, step as

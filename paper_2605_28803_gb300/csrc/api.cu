@@ -30,6 +30,9 @@ struct qvla_layer {
   int grouped = 0;            // the table holds one scale per (step, channel group)
   int group = 128, G = 1;     // channels per scale group (max(128, had_block)) and groups per row
   float* wgcorr = nullptr;    // device [N][G]: 8 * (sum of row n's codes over group g), non-gated layers
+  int32_t* rperm = nullptr;   // device [K]: online permutation (identity when only U is given)
+  float* rrot = nullptr;      // device [K/rblock][rblock][rblock]: online U_b blocks, float32
+  int rblock = 0;             // 0: the activations arrive in the P.U basis (no online rotation)
 };
 
 namespace {
@@ -90,6 +93,11 @@ int num_sms(int device) {
 }
 
 size_t round256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+
+// bytes of an [M][K] activation tensor of the layer's input dtype
+size_t rotated_bytes(const qvla_layer* L, int M) {
+  return static_cast<size_t>(M) * L->K * (L->xdt == QVLA_F32 ? 4 : 2);
+}
 
 qvla_status check_rows(int M) {
   if (M < 0 || M > (1 << 20)) return fail(QVLA_ERR_INVALID_ARG, "M=%d outside [0, 2^20]", M);
@@ -349,6 +357,8 @@ qvla_status qvla_layer_destroy(qvla_layer* L) {
   cudaFree(L->wgcorr);
   cudaFree(L->bias);
   cudaFree(L->table);
+  cudaFree(L->rperm);
+  cudaFree(L->rrot);
   delete L;
   return QVLA_OK;
 }
@@ -408,6 +418,73 @@ qvla_status qvla_layer_scale_groups(const qvla_layer* L, int* G, int* group) {
   return QVLA_OK;
 }
 
+qvla_status qvla_layer_set_online_rotation(qvla_layer* L, const int32_t* perm, const double* rot, int rot_block) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  const int K = L->K;
+  if (!perm && !rot) {  // back to activations that arrive in the P.U basis
+    QVLA_CUDA(cudaDeviceSynchronize(), "synchronise before freeing the online rotation");
+    cudaFree(L->rperm);
+    cudaFree(L->rrot);
+    L->rperm = nullptr;
+    L->rrot = nullptr;
+    L->rblock = 0;
+    return QVLA_OK;
+  }
+  if (!rot) rot_block = 16;  // a permutation alone: identity blocks
+  if (rot_block != 16 && rot_block != 32 && rot_block != 64)
+    return fail(QVLA_ERR_UNSUPPORTED, "rot_block=%d: the online rotation takes blocks of 16, 32 or 64 channels", rot_block);
+  if (K % rot_block != 0) return fail(QVLA_ERR_INVALID_ARG, "rot_block=%d does not divide K=%d", rot_block, K);
+  std::vector<int32_t> hp(K);
+  if (perm) {
+    std::vector<char> seen(K, 0);
+    for (int k = 0; k < K; ++k) {
+      const int32_t v = perm[k];
+      if (v < 0 || v >= K || seen[v]) return fail(QVLA_ERR_INVALID_ARG, "perm is not a permutation of [0, K)");
+      seen[v] = 1;
+      hp[k] = v;
+    }
+  } else {
+    for (int k = 0; k < K; ++k) hp[k] = k;
+  }
+  const size_t nrot = static_cast<size_t>(K) * rot_block;  // (K / rot_block) blocks of rot_block^2
+  std::vector<float> hr(nrot, 0.0f);
+  for (size_t i = 0; i < nrot; ++i) {
+    if (rot) {
+      if (!std::isfinite(rot[i])) return fail(QVLA_ERR_INVALID_ARG, "rot holds a non-finite entry");
+      hr[i] = static_cast<float>(rot[i]);
+    } else {
+      const size_t e = i % (static_cast<size_t>(rot_block) * rot_block);
+      hr[i] = (e / rot_block == e % rot_block) ? 1.0f : 0.0f;
+    }
+  }
+  QVLA_CUDA(cudaDeviceSynchronize(), "synchronise before replacing the online rotation");
+  cudaFree(L->rperm);
+  cudaFree(L->rrot);
+  L->rperm = nullptr;
+  L->rrot = nullptr;
+  L->rblock = 0;
+  QVLA_CUDA(cudaMalloc(&L->rperm, hp.size() * sizeof(int32_t)), "online permutation allocation");
+  QVLA_CUDA(cudaMalloc(&L->rrot, hr.size() * sizeof(float)), "online rotation allocation");
+  QVLA_CUDA(cudaMemcpy(L->rperm, hp.data(), hp.size() * sizeof(int32_t), cudaMemcpyHostToDevice), "online permutation upload");
+  QVLA_CUDA(cudaMemcpy(L->rrot, hr.data(), hr.size() * sizeof(float), cudaMemcpyHostToDevice), "online rotation upload");
+  L->rblock = rot_block;
+  return QVLA_OK;
+}
+
+qvla_status qvla_online_rotate(const qvla_layer* L, const void* x, int M, void* out, void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_rows(M)) return s;
+  if (!L->rblock) return fail(QVLA_ERR_INVALID_ARG, "the layer has no online rotation");
+  if (M == 0) return QVLA_OK;
+  if (!x || !out) return fail(QVLA_ERR_INVALID_ARG, "x and out must not be NULL");
+  QVLA_CUDA(qvla::launch_block_rotate(x, L->xdt, M, L->K, L->rperm, L->rrot, L->rblock, out,
+                                      static_cast<cudaStream_t>(stream)),
+            "online rotation launch");
+  return QVLA_OK;
+}
+
 qvla_status qvla_layer_info(const qvla_layer* L, int* N, int* K, int* had_block, int* T) {
   g_last_error.clear();
   if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
@@ -439,6 +516,8 @@ qvla_status qvla_rotate_quantize(const qvla_layer* L, const void* x, int M, int 
   if (qvla_status s = resolve_step(L, step, &ss)) return s;
   if (ss && L->grouped)
     return fail(QVLA_ERR_UNSUPPORTED, "per-group step scales run through qvla_w4a4_linear only (codes alone have no single scale)");
+  if (L->rblock)
+    return fail(QVLA_ERR_UNSUPPORTED, "the layer's online rotation runs in qvla_w4a4_linear / qvla_linear_quantize");
   if (M == 0) return QVLA_OK;
   if (!x || !xq || !xscale) return fail(QVLA_ERR_INVALID_ARG, "x, xq and xscale must not be NULL");
   if (!aligned16(x) || !aligned16(xq)) return fail(QVLA_ERR_INVALID_ARG, "x and xq must be 16-byte aligned");
@@ -538,7 +617,7 @@ size_t qvla_linear_workspace_bytes(const qvla_layer* L, int M) {
   // the codes travel between the two kernels as one operand byte each; then the scales, the
   // code sums and the per-group code sums (used with per-group step scales)
   return round256(static_cast<size_t>(M) * L->K) + round256(static_cast<size_t>(M) * 4) * 2 +
-         round256(static_cast<size_t>(M) * L->G * 4);
+         round256(static_cast<size_t>(M) * L->G * 4) + (L->rblock ? round256(rotated_bytes(L, M)) : 0);
 }
 
 namespace {
@@ -547,6 +626,7 @@ struct LinearWorkspace {
   float* xscale;     // [M]
   int32_t* xsum;     // [M]
   int32_t* xgsum;    // [M][G]
+  void* xrot;        // [M][K] x . P . BlockDiag(U_b) in the activation dtype (layers with an online rotation)
 };
 
 qvla_status carve_workspace(const qvla_layer* L, int M, void* workspace, size_t workspace_bytes, LinearWorkspace* w) {
@@ -560,6 +640,20 @@ qvla_status carve_workspace(const qvla_layer* L, int M, void* workspace, size_t 
   w->xscale = reinterpret_cast<float*>(ws + round256(static_cast<size_t>(M) * L->K));
   w->xsum = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(w->xscale) + round256(static_cast<size_t>(M) * 4));
   w->xgsum = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(w->xsum) + round256(static_cast<size_t>(M) * 4));
+  w->xrot = reinterpret_cast<uint8_t*>(w->xgsum) + round256(static_cast<size_t>(M) * L->G * 4);
+  return QVLA_OK;
+}
+
+// The activations the quantiser sees: x itself, or x . P . BlockDiag(U_b) formed in the workspace
+// when the layer carries an online rotation.
+qvla_status online_input(const qvla_layer* L, const void* x, int M, const LinearWorkspace& w, void* stream,
+                         const void** xin) {
+  *xin = x;
+  if (!L->rblock) return QVLA_OK;
+  QVLA_CUDA(qvla::launch_block_rotate(x, L->xdt, M, L->K, L->rperm, L->rrot, L->rblock, w.xrot,
+                                      static_cast<cudaStream_t>(stream)),
+            "online rotation launch");
+  *xin = w.xrot;
   return QVLA_OK;
 }
 }  // namespace
@@ -578,7 +672,9 @@ qvla_status qvla_linear_quantize(const qvla_layer* L, const void* x, int M, int 
   if (!aligned16(x)) return fail(QVLA_ERR_INVALID_ARG, "x must be 16-byte aligned");
   LinearWorkspace w;
   if (qvla_status s = carve_workspace(L, M, workspace, workspace_bytes, &w)) return s;
-  return launch_rq(x, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr, stream, 1);
+  const void* xin = nullptr;
+  if (qvla_status s = online_input(L, x, M, w, stream, &xin)) return s;
+  return launch_rq(xin, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr, stream, 1);
 }
 
 qvla_status qvla_linear_gemm(const qvla_layer* L, const void* workspace, size_t workspace_bytes, int M, void* y,
@@ -606,13 +702,16 @@ qvla_status qvla_w4a4_linear(const qvla_layer* L, const void* x, int M, int step
   if (!aligned16(x) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "x and y must be 16-byte aligned");
   LinearWorkspace w;
   if (qvla_status s = carve_workspace(L, M, workspace, workspace_bytes, &w)) return s;
+  const void* xin = nullptr;
+  if (qvla_status s = online_input(L, x, M, w, stream, &xin)) return s;
   if (ss && L->grouped) {  // per-group step scales: per-group codes and sums, promoted per group
-    if (qvla_status s = launch_rq(x, L->xdt, M, L->K, L->had_block, 1, ss, w.xb, w.xscale, nullptr, nullptr, stream, 1,
+    if (qvla_status s = launch_rq(xin, L->xdt, M, L->K, L->had_block, 1, ss, w.xb, w.xscale, nullptr, nullptr, stream, 1,
                                   L->group, w.xgsum))
       return s;
     return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream, ss, w.xgsum);
   }
-  if (qvla_status s = launch_rq(x, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr, stream, 1))
+  if (qvla_status s = launch_rq(xin, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr,
+                                stream, 1))
     return s;
   return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream);
 }
@@ -665,6 +764,8 @@ qvla_status qvla_w4a8_linear(const qvla_layer* L, const void* x, int M, int step
   const float* ss = nullptr;
   if (qvla_status s = resolve_step(L, step, &ss)) return s;
   if (ss && L->grouped) return fail(QVLA_ERR_UNSUPPORTED, "per-group step scales are for int4 activation codes");
+  if (L->rblock)
+    return fail(QVLA_ERR_UNSUPPORTED, "the layer's online rotation runs in qvla_w4a4_linear / qvla_linear_quantize");
   if (M == 0) return QVLA_OK;
   if (!x || !y) return fail(QVLA_ERR_INVALID_ARG, "x and y must not be NULL");
   if (!aligned16(x) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "x and y must be 16-byte aligned");

@@ -39,6 +39,13 @@ cudaError_t launch_rotate_quant(const RotQuantArgs& a);
 // or null (cleared, then the codes' row sums added).
 cudaError_t launch_a8_planes(const int8_t* xq, int M, int K, uint8_t* planes, int32_t* xsum, cudaStream_t stream);
 
+// ---- online x . P . BlockDiag(U_b) (block_rotate.cu) ----
+// x, out: device [M][K] of activation dtype xdt (0 f16, 1 bf16, 2 f32); perm: device int32 [K]
+// (identity when the layer has none); rot: device float32 [K/block][block][block], 16-byte
+// aligned; block in {16, 32, 64} dividing K.
+cudaError_t launch_block_rotate(const void* x, int xdt, int M, int K, const int32_t* perm, const float* rot, int block,
+                                void* out, cudaStream_t stream);
+
 // ---- W4A4 GEMM + epilogue (gemm.cu) ----
 struct GemmArgs {
   const uint8_t* xq;       // device activations, by x_bytes:

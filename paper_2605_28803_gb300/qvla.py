@@ -36,6 +36,8 @@ SIGNATURES = {
     "qvla_set_step_scales": (_I, [_P, _P, _I]),
     "qvla_set_step_group_scales": (_I, [_P, _P, _I, _I]),
     "qvla_layer_scale_groups": (_I, [_P, _P, _P]),
+    "qvla_layer_set_online_rotation": (_I, [_P, _P, _P, _I]),
+    "qvla_online_rotate": (_I, [_P, _P, _I, _P, _P]),
     "qvla_rotated_absmax_groups": (_I, [_P, _I, _I, _I, _I, _P, _P]),
     "qvla_layer_info": (_I, [_P, _P, _P, _P, _P]),
     "qvla_rotate_quantize": (_I, [_P, _P, _I, _I, _P, _P, _P, _P]),
@@ -187,6 +189,18 @@ def qvla_set_step_group_scales(layer: Layer, scales: np.ndarray) -> None:
     if arr.ndim != 2:
         raise ValueError("scales must be [T, G]")
     _check(_lib.qvla_set_step_group_scales(layer.handle, _ptr(arr), arr.shape[0], arr.shape[1]))
+
+
+def qvla_layer_set_online_rotation(layer: Layer, perm=None, rot=None, rot_block: int = 0) -> None:
+    """Online x . P . BlockDiag(U_b) ahead of the layer's quantiser (perm int32 [K], rot float64
+    [K/rot_block, rot_block, rot_block]); both None removes it."""
+    p = None if perm is None else np.ascontiguousarray(perm, dtype=np.int32)
+    r = None if rot is None else np.ascontiguousarray(rot, dtype=np.float64)
+    _check(_lib.qvla_layer_set_online_rotation(layer.handle, _ptr(p), _ptr(r), int(rot_block)))
+
+
+def qvla_online_rotate(layer: Layer, x, M: int, out, stream=None) -> None:
+    _check(_lib.qvla_online_rotate(layer.handle, _ptr(x), M, _ptr(out), _stream(stream)))
 
 
 def qvla_layer_scale_groups(layer: Layer):

@@ -68,6 +68,12 @@ def test_validation_precedes_any_device_work():
         Q.qvla_rotated_absmax(None, Q.F16, 1 << 21, 128, 1, None)
 
 
+def test_online_rotation_entry_points_reject_a_null_layer():
+    # argument checks that need no GPU: both entry points report a NULL layer
+    assert Q._lib.qvla_layer_set_online_rotation(None, None, None, 64) == 1
+    assert Q._lib.qvla_online_rotate(None, None, 4, None, None) == 1
+
+
 def _host_pack(w, wdt, had, rot=None, rot_block=0, perm=None):
     N, K = w.shape
     wq = np.zeros((N, K // 2), np.uint8)
