@@ -60,13 +60,31 @@ __global__ void __launch_bounds__(kBrThreads) block_rotate_kernel(const T* __res
   const int m0 = blockIdx.y * kRows;
   const int t = threadIdx.x;
 
+  // every load is issued before any is used: thread t gathers channel perm[b kB + t % kB] of rows
+  // t / kB, t / kB + kRStep, ..., and copies float4 t, t + kBrThreads, ... of U_b
+  static_assert(kBrThreads % kB == 0, "a thread's gathered channel is fixed");
+  constexpr int kRStep = kBrThreads / kB;
+  constexpr int kPer = kRows / kRStep;                     // gathered values per thread
+  constexpr int kU4 = kB * kB / 4;                         // float4 of U_b
+  constexpr int kUPer = (kU4 + kBrThreads - 1) / kBrThreads;
   const float4* usrc = reinterpret_cast<const float4*>(rot + static_cast<size_t>(b) * kB * kB);
-  for (int i = t; i < kB * kB / 4; i += kBrThreads) reinterpret_cast<float4*>(su)[i] = __ldg(usrc + i);
-  for (int e = t; e < kRows * kB; e += kBrThreads) {
-    const int r = e / kB, i = e - r * kB;
-    const int m = m0 + r;
-    sz[r][i] = m < M ? load_f(x + static_cast<size_t>(m) * K + __ldg(perm + b * kB + i)) : 0.0f;
+  float4 uv[kUPer];
+#pragma unroll
+  for (int j = 0; j < kUPer; ++j)
+    if (kU4 % kBrThreads == 0 || t + j * kBrThreads < kU4) uv[j] = __ldg(usrc + t + j * kBrThreads);
+  const int gi = t % kB, gr = t / kB;
+  const int col = __ldg(perm + b * kB + gi);
+  float gv[kPer];
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) {
+    const int m = m0 + gr + j * kRStep;
+    gv[j] = m < M ? load_f(x + static_cast<size_t>(m) * K + col) : 0.0f;
   }
+#pragma unroll
+  for (int j = 0; j < kUPer; ++j)
+    if (kU4 % kBrThreads == 0 || t + j * kBrThreads < kU4) reinterpret_cast<float4*>(su)[t + j * kBrThreads] = uv[j];
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) sz[gr + j * kRStep][gi] = gv[j];
   __syncthreads();
 
   const int rg = t >> 4, cg = t & 15;  // rows 4 rg .. 4 rg + 3, columns cg + 16 j
