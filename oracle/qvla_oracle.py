@@ -39,6 +39,8 @@ Readings of the paper that this file fixes (each is also listed in the design no
   R6  Packed int4: byte j of a row holds code 2j in its low nibble and code 2j+1 in
       its high nibble, each as a 4-bit two's-complement integer.
   R7  The down-projection glue of the gated MLP is gelu_tanh(gate) * up.
+  R20 The q999 peak statistic is the 0.999 quantile of |y| with linear interpolation between
+      order statistics.
   R14 The zigzag deals the energy-sorted channels (ties: lower index first) forwards in even
       rounds and backwards in odd ones; Eq. 5's W' = P^T R_hat^T W is read as the fold that
       keeps X W unchanged, R_hat^T P^T W.
@@ -457,7 +459,8 @@ def robust_peak(y: np.ndarray, estimator: str = "absmax") -> np.float32:
     """sigma_hat of Eq. 6: a robust peak estimate of a calibration tensor.
 
     "absmax" is max|y|; "q999" is the 99.9th percentile of |y| (the appendix on per-step
-    scaling measures q999).  Returned as float32.
+    scaling measures q999), read as the 0.999 quantile with linear interpolation between order
+    statistics (reading R20).  Returned as float32.
     """
     a = np.abs(np.asarray(y, dtype=np.float64)).ravel()
     if estimator == "absmax":
@@ -560,7 +563,8 @@ def w4a4_linear(x: np.ndarray, w_codes: np.ndarray, w_scale: np.ndarray, had_blo
 # --------------------------------------------------------------------------------------
 
 def gelu_tanh(x: np.ndarray) -> np.ndarray:
-    """GELU, tanh form, float64."""
+    """GELU, tanh form, float64: x/2 (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3))), the activation
+    of the gated MLP of the Pi-0.5 / PaliGemma backbone (Sec. 5.1; reading R7)."""
     x = np.asarray(x, dtype=np.float64)
     return 0.5 * x * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (x + 0.044715 * x ** 3)))
 

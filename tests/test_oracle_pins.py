@@ -12,6 +12,7 @@ import math
 import numpy as np
 import pytest
 import scipy.linalg
+import scipy.special
 import torch
 
 from oracle import qvla_oracle as O
@@ -552,6 +553,49 @@ def check_grouped_calibration(o):
             assert np.abs(q[:, g * 128:(g + 1) * 128]).max() == 7
 
 
+def check_gelu_golden(o):
+    """The tanh-form GELU of the gated MLP glue (reading R7) at hand-worked points
+    (tests/golden/gelu_worked.txt), and the glue h = gelu(gate) * up."""
+    g = read_golden("gelu_worked.txt")
+    x = np.array([float(v) for v in g["x"]])
+    want = np.array([float(v) for v in g["gelu"]])
+    assert np.allclose(o.gelu_tanh(x), want, rtol=0, atol=5e-15)
+    gate = np.array([float(v) for v in g["gate"]])
+    up = np.array([float(v) for v in g["up"]])
+    assert np.allclose(o.gated_glue(gate, up), np.array([float(v) for v in g["h"]]), rtol=0, atol=5e-15)
+
+
+def check_gelu_library_and_identities(o):
+    """gelu_tanh equals torch's GELU with approximate='tanh' (float64) on a grid over +-10;
+    its odd part is x/2 (gelu(x) - gelu(-x) = x for the tanh form); it tends to x above and to
+    0 below; it differs from the exact erf form (the other GELU) by more than rounding."""
+    x = np.linspace(-10.0, 10.0, 4001)
+    lib = torch.nn.functional.gelu(torch.from_numpy(x), approximate="tanh").numpy()
+    assert np.allclose(o.gelu_tanh(x), lib, rtol=1e-14, atol=1e-15)
+    assert np.allclose(o.gelu_tanh(x) - o.gelu_tanh(-x), x, rtol=0, atol=1e-13)
+    assert abs(o.gelu_tanh(np.array([30.0]))[0] - 30.0) < 1e-12 and abs(o.gelu_tanh(np.array([-30.0]))[0]) < 1e-12
+    erf_form = torch.nn.functional.gelu(torch.from_numpy(x), approximate="none").numpy()
+    assert np.abs(o.gelu_tanh(x) - erf_form).max() > 1e-4
+    rng = np.random.default_rng(44)
+    gate, up = rng.standard_normal(64) * 3, rng.standard_normal(64)
+    lib_h = torch.nn.functional.gelu(torch.from_numpy(gate), approximate="tanh").numpy() * up
+    assert np.allclose(o.gated_glue(gate, up), lib_h, rtol=1e-14, atol=1e-15)
+
+
+def check_q999_golden(o):
+    """The q999 peak statistic (Eq. 6's sigma_hat as the appendix measures it) on a hand-worked
+    case (tests/golden/q999_worked.txt): the 0.999 quantile of |y| with linear interpolation."""
+    g = read_golden("q999_worked.txt")
+    n = int(g["n"][0])
+    y = np.array([(-1) ** i * i for i in range(n)], dtype=np.float64)
+    assert o.robust_peak(y, "q999") == np.float32(float(g["q999"][0]))
+    assert o.robust_peak(y, "absmax") == np.float32(float(g["absmax"][0]))
+    # the same statistic through the calibration of a per-step table: sigma_hat / 7 of the rotated
+    # activations; with b = 1 (no rotation) the activations are y itself
+    tab = o.calibrate_step_table([y.reshape(8, n // 8)], 1, "q999")
+    assert tab[0] == np.float32(998.001) / np.float32(7)
+
+
 PINS = {f.__name__: f for f in [
     check_hadamard_matches_scipy, check_hadamard_orthogonal, check_hadamard_golden,
     check_rotate_matches_library_blockdiag, check_rotate_linf_bound, check_rotation_invariance,
@@ -564,6 +608,7 @@ PINS = {f.__name__: f for f in [
     check_gptq_two_columns_closed_form, check_gptq_identity_hessian_is_rtn, check_gptq_matches_obq_sequential,
     check_gptq_block_invariance_and_loss, check_gptq_dead_column,
     check_grouped_equal_scales_reduce_to_per_tensor, check_grouped_linear_bruteforce, check_grouped_calibration,
+    check_gelu_golden, check_gelu_library_and_identities, check_q999_golden,
 ]}
 
 
@@ -746,6 +791,46 @@ def _mut_group_size_fixed_128(k, had_block):
     return 128
 
 
+def _mut_gelu_coefficient(x):
+    x = np.asarray(x, dtype=np.float64)
+    return 0.5 * x * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (x + 0.04715 * x ** 3)))
+
+
+def _mut_gelu_no_sqrt_2_over_pi(x):
+    x = np.asarray(x, dtype=np.float64)
+    return 0.5 * x * (1.0 + np.tanh(x + 0.044715 * x ** 3))
+
+
+def _mut_gelu_erf_form(x):
+    x = np.asarray(x, dtype=np.float64)
+    return 0.5 * x * (1.0 + scipy.special.erf(x / math.sqrt(2.0)))
+
+
+def _mut_glue_swapped(gate, up):
+    return O.gelu_tanh(up) * np.asarray(gate, dtype=np.float64)
+
+
+def _mut_q999_at_099(y, estimator="absmax"):
+    a = np.abs(np.asarray(y, dtype=np.float64)).ravel()
+    if estimator == "q999":
+        return np.float32(np.quantile(a, 0.99))
+    return np.float32(a.max(initial=0.0))
+
+
+def _mut_q999_nearest(y, estimator="absmax"):
+    a = np.abs(np.asarray(y, dtype=np.float64)).ravel()
+    if estimator == "q999":
+        return np.float32(np.quantile(a, 0.999, method="nearest"))
+    return np.float32(a.max(initial=0.0))
+
+
+def _mut_q999_signed(y, estimator="absmax"):
+    a = np.asarray(y, dtype=np.float64).ravel()
+    if estimator == "q999":
+        return np.float32(np.quantile(a, 0.999))
+    return np.float32(np.abs(a).max(initial=0.0))
+
+
 MUTANTS = {
     "hadamard_wrong_order": ("sylvester_hadamard", _mut_hadamard_order),
     "rotate_unnormalised": ("block_hadamard_rotate", _mut_rotate_unnormalised),
@@ -773,6 +858,13 @@ MUTANTS = {
     "grouped_scale_shifted_one_channel": ("quantize_activations_per_step_grouped", _mut_group_of_next_channel),
     "grouped_scale_first_group_only": ("quantize_activations_per_step_grouped", _mut_group_first_only),
     "group_size_ignores_hadamard_block": ("step_group_size", _mut_group_size_fixed_128),
+    "gelu_cubic_coefficient": ("gelu_tanh", _mut_gelu_coefficient),
+    "gelu_without_sqrt_2_over_pi": ("gelu_tanh", _mut_gelu_no_sqrt_2_over_pi),
+    "gelu_erf_form": ("gelu_tanh", _mut_gelu_erf_form),
+    "glue_gate_and_up_swapped": ("gated_glue", _mut_glue_swapped),
+    "q999_at_0_99": ("robust_peak", _mut_q999_at_099),
+    "q999_nearest_rank": ("robust_peak", _mut_q999_nearest),
+    "q999_without_abs": ("robust_peak", _mut_q999_signed),
 }
 
 
