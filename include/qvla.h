@@ -183,7 +183,8 @@ qvla_status qvla_set_step_group_scales(qvla_layer* layer, const float* scales, i
  *   rot        host float64 [K/rot_block][rot_block][rot_block], row-major U_b (uploaded as
  *              float32), or NULL (U = I; perm alone).  Orthogonality is the caller's promise.
  *   rot_block  16, 32 or 64 (QVLA_ERR_UNSUPPORTED otherwise), dividing K.
- * perm == NULL and rot == NULL removes the online rotation.  Synchronous. */
+ * perm == NULL and rot == NULL removes the online rotation.  Synchronous; the layer's device
+ * must be current (QVLA_ERR_INVALID_ARG otherwise). */
 qvla_status qvla_layer_set_online_rotation(qvla_layer* layer, const int32_t* perm, const double* rot, int rot_block);
 
 /* The layer's online rotation alone: out = x . P . BlockDiag(U_b) as above (x, out device
@@ -287,8 +288,11 @@ qvla_status qvla_linear_gemm(const qvla_layer* layer, const void* workspace, siz
  * makes no cudaMalloc/cudaFree and calls no allocating library routine.  Its first call on each
  * device looks up the array's device address with that device current; make that first call
  * before any stream capture.  The scratch must hold qvla_linear_workspace_bytes(layer, M)
- * bytes (the codes [M][K] as operand bytes, scales and code sums); larger requests fail with
- * QVLA_ERR_UNSUPPORTED and enqueue nothing.  Every call shares the one array and leaves the
+ * bytes, each part rounded up to a multiple of 256: the codes as operand bytes (M x K), the
+ * scales and the code sums (M x 4 each), the per-group code sums (M x G x 4, G = K / max(128,
+ * had_block)) and, for a layer with an online rotation, x . P . BlockDiag(U_b) (M x K elements
+ * of the activation dtype).  Larger requests fail with QVLA_ERR_UNSUPPORTED and enqueue
+ * nothing.  The layer must live on the current device (QVLA_ERR_INVALID_ARG otherwise).  Every call shares the one array and leaves the
  * last call's contents in it; each call overwrites all it reads, so nothing needs clearing
  * in between.  Two calls whose kernels overlap on the GPU (different streams or threads, on
  * the same device) race on the array: issue them on one stream.

@@ -128,6 +128,16 @@ qvla_status launch_rq(const void* x, int xdt, int M, int K, int had_block, int m
   return QVLA_OK;
 }
 
+// A layer's buffers live on the device that was current when it was created; its kernels must be
+// launched with that device current.
+qvla_status check_layer_device(const qvla_layer* L) {
+  int dev = 0;
+  QVLA_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
+  if (dev != L->device)
+    return fail(QVLA_ERR_INVALID_ARG, "the current device is %d but the layer lives on device %d", dev, L->device);
+  return QVLA_OK;
+}
+
 qvla_status resolve_step(const qvla_layer* layer, int step, const float** step_scale) {
   if (step == -1) {
     *step_scale = nullptr;
@@ -421,6 +431,7 @@ qvla_status qvla_layer_scale_groups(const qvla_layer* L, int* G, int* group) {
 qvla_status qvla_layer_set_online_rotation(qvla_layer* L, const int32_t* perm, const double* rot, int rot_block) {
   g_last_error.clear();
   if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_layer_device(L)) return s;
   const int K = L->K;
   if (!perm && !rot) {  // back to activations that arrive in the P.U basis
     QVLA_CUDA(cudaDeviceSynchronize(), "synchronise before freeing the online rotation");
@@ -823,6 +834,7 @@ extern "C" {
 qvla_status qvla_w4a4_linear_noalloc(const qvla_layer* L, const void* x, int M, int step, void* y, void* stream) {
   g_last_error.clear();
   if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_layer_device(L)) return s;  // the scratch looked up is the current device's
   if (qvla_status s = check_rows(M)) return s;
   const size_t need = qvla_linear_workspace_bytes(L, M);
   if (need > QVLA_NOALLOC_SCRATCH_BYTES)

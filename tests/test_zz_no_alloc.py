@@ -73,3 +73,20 @@ def test_noalloc_rejects_more_rows_than_its_scratch_holds():
         Q.qvla_w4a4_linear_noalloc(layer, x, too_many, -1, y, G.stream())
     assert e.value.status == 2 and "scratch" in str(e.value)
     layer.close()
+
+
+def test_noalloc_counts_the_online_rotation_in_its_scratch():
+    # A layer with an online x.P.BlockDiag(U_b) keeps x' in the scratch as well: 2000 rows of
+    # K = 2048 fit without it (operand bytes and sums) but not with 2000 x 2048 bf16 values more.
+    K, N, M = 2048, 256, 2000
+    case = W.sweep_linear(16, K, N, seed=24, xdtype="bf16", ydtype="bf16")
+    layer = _layer(case, "bf16", "bf16")
+    assert Q.qvla_linear_workspace_bytes(layer, M) <= Q.NOALLOC_SCRATCH_BYTES
+    Q.qvla_layer_set_online_rotation(layer, perm=np.arange(K - 1, -1, -1, dtype=np.int32), rot=None, rot_block=16)
+    assert Q.qvla_linear_workspace_bytes(layer, M) > Q.NOALLOC_SCRATCH_BYTES
+    x = torch.zeros(M, K, dtype=torch.bfloat16, device=G.DEV)
+    y = torch.zeros(M, N, dtype=torch.bfloat16, device=G.DEV)
+    with pytest.raises(Q.QvlaError) as e:
+        Q.qvla_w4a4_linear_noalloc(layer, x, M, -1, y, G.stream())
+    assert e.value.status == 2 and "scratch" in str(e.value)
+    layer.close()
