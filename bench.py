@@ -62,6 +62,7 @@ def parse():
     ap.add_argument("--sets", type=int, default=3, help="rotating weight+activation sets (working set > L2)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="CPU-baseline sample budget")
     ap.add_argument("--no-stacks", action="store_true", help="skip the DiT and backbone stack legs")
+    ap.add_argument("--no-sweep", action="store_true", help="skip the single-layer and sweep legs")
     return ap.parse_args()
 
 
@@ -109,23 +110,82 @@ def max_over_ranks(world, value: float, device) -> float:
 # --------------------------------------------------------------------------------------
 
 def peaks():
+    """Measured roofline denominators: E4M3 tensor rate as the measured bf16 GEMM rate times the
+    nominal E4M3/bf16 ratio, burst (a kernel timed alone) and sustained (inside a long loop),
+    and the HBM copy bandwidth."""
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
         d = json.load(open(p))
-        return d["bf16_tflops_sustained"] * FP8_OVER_BF16, d["hbm_gbs"], "measured"
-    return 1700.0 * FP8_OVER_BF16, 6800.0, "fallback"
+        return {"tflops": d["bf16_tflops"] * FP8_OVER_BF16, "tflops_sustained": d["bf16_tflops_sustained"] * FP8_OVER_BF16,
+                "gbs": d["hbm_gbs"], "src": "measured"}
+    return {"tflops": 1900.0 * FP8_OVER_BF16, "tflops_sustained": 1700.0 * FP8_OVER_BF16, "gbs": 6800.0, "src": "fallback"}
+
+
+class _Nvml:
+    """The few NVML queries the clock record needs, through ctypes (reading only)."""
+    SM = 1  # NVML_CLOCK_SM
+    REASONS = {0x8: "hw_slowdown", 0x40: "hw_thermal_slowdown", 0x20: "sw_thermal_slowdown", 0x4: "sw_power_cap"}
+
+    def __init__(self, device_index: int):
+        import ctypes
+
+        self.c = ctypes
+        lib = ctypes.CDLL("libnvidia-ml.so.1")
+        if lib.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit failed")
+        self.lib = lib
+        self.h = ctypes.c_void_p()
+        props = torch.cuda.get_device_properties(device_index)
+        bus = None
+        if all(hasattr(props, a) for a in ("pci_domain_id", "pci_bus_id", "pci_device_id")):
+            bus = f"{props.pci_domain_id:08x}:{props.pci_bus_id:02x}:{props.pci_device_id:02x}.0".encode()
+        if bus is None or lib.nvmlDeviceGetHandleByPciBusId_v2(bus, ctypes.byref(self.h)) != 0:
+            if lib.nvmlDeviceGetHandleByIndex_v2(device_index, ctypes.byref(self.h)) != 0:
+                raise OSError("no NVML handle")
+        self.reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            lib.nvmlDeviceGetCurrentClocksThrottleReasons
+
+    def sample(self):
+        c = self.c
+        mhz, mx, mw, rs = c.c_uint(), c.c_uint(), c.c_uint(), c.c_ulonglong()
+        if self.lib.nvmlDeviceGetClockInfo(self.h, self.SM, c.byref(mhz)) != 0:
+            return None
+        self.lib.nvmlDeviceGetMaxClockInfo(self.h, self.SM, c.byref(mx))
+        self.lib.nvmlDeviceGetPowerUsage(self.h, c.byref(mw))
+        self.reasons_fn(self.h, c.byref(rs))
+        reasons = [name for bit, name in self.REASONS.items() if rs.value & bit]
+        return float(mhz.value), float(mx.value), mw.value / 1000.0, reasons
 
 
 class ClockSampler:
+    """SM clocks, power and slowdown reasons sampled every few milliseconds from a host thread
+    while the GPU runs; each sample is tagged with whether the timed region was running (its
+    start event had completed and its end event had not).  NVML through ctypes; nvidia-smi at
+    200 ms when NVML cannot be opened."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
               "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
               "clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
-        self.proc = None
+    def __init__(self, gpu_index: int, period_s: float = 0.002):
         self.gpu = gpu_index
+        self.period = period_s
+        self.samples = []
+        self.region = None  # (start event, end event) of the timed region
+        self.proc = self.thread = self.nvml = None
+        self.stop_flag = False
 
-    def start(self):
+    def start(self, region=None):
+        import threading
+
+        self.region = region
+        try:
+            self.nvml = _Nvml(self.gpu)
+        except (OSError, AttributeError):
+            self.nvml = None
+        if self.nvml is not None:
+            self.thread = threading.Thread(target=self._poll, daemon=True)
+            self.thread.start()
+            return
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
                                           "--format=csv,noheader,nounits", "-lms", "200"],
@@ -133,30 +193,64 @@ class ClockSampler:
         except (OSError, FileNotFoundError):
             self.proc = None
 
-    def stop(self):
-        if self.proc is None:
-            return None
+    def _in_region(self):
+        if self.region is None:
+            return False
+        a, b = self.region
+        try:
+            return a.query() and not b.query()
+        except RuntimeError:
+            return False
+
+    def _poll(self):
+        while not self.stop_flag:
+            r = self.nvml.sample()
+            if r is not None:
+                self.samples.append(r + (self._in_region(),))
+            time.sleep(self.period)
+
+    def _smi_rows(self):
         self.proc.terminate()
         try:
             out, _ = self.proc.communicate(timeout=5)
         except subprocess.TimeoutExpired:
             self.proc.kill()
             out, _ = self.proc.communicate()
-        rows = [r.split(", ") for r in out.strip().splitlines() if r.strip()]
-        sm, mx, reasons = [], 0.0, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for r in rows:
+        rows = []
+        for r in (r.split(", ") for r in out.strip().splitlines() if r.strip()):
             try:
-                sm.append(float(r[1]))
-                mx = max(mx, float(r[2]))
+                rows.append((float(r[1]), float(r[2]), float(r[3]),
+                             [n for n, v in zip(names, r[5:9]) if v.strip().lower() == "active"], False))
             except (ValueError, IndexError):
                 continue
-            for name, v in zip(names, r[5:9]):
-                if v.strip().lower() == "active":
-                    reasons.add(name)
-        if not sm:
+        return rows
+
+    def stop(self):
+        if self.thread is not None:
+            self.stop_flag = True
+            self.thread.join(timeout=5)
+            rows, how = self.samples, "NVML every 2 ms"
+        elif self.proc is not None:
+            rows, how = self._smi_rows(), "nvidia-smi every 200 ms"
+        else:
             return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+        return self.summarize(rows, how)
+
+    @staticmethod
+    def summarize(rows, how):
+        """rows: (sm MHz, max SM MHz, watts, [slowdown reasons], inside the timed region)."""
+        if not rows:
+            return None
+        inside = [r for r in rows if r[4]]
+        use = inside if len(inside) >= 3 else rows
+        reasons = sorted({n for r in use for n in r[3]})
+        return {"sm_mhz": statistics.median(r[0] for r in use), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "power_w_max": round(max(r[2] for r in use), 1), "samples": len(use),
+                "samples_in_timed_region": len(inside),
+                "window": ("the timed region" if use is inside else
+                           "back-to-back steps bracketing the timed region (too short to sample alone)"),
+                "how": how}
 
 
 def gemm_traffic():
@@ -234,10 +328,14 @@ def run_ours(args):
         if ev is not None:
             ev[4].record(stream)
 
+    w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    w0.record(stream)
     for i in range(args.warmup):
         step(sets[i % args.sets])
+    w1.record(stream)
     torch.cuda.synchronize()
     Q.qvla_check_device(stream)
+    warm_ms = w0.elapsed_time(w1) / max(1, args.warmup)
 
     # ---- device-timed region: inputs resident in HBM ----
     K = args.steps
@@ -246,14 +344,22 @@ def run_ours(args):
     EVERY = 8
     evs = {i: [torch.cuda.Event(enable_timing=True) for _ in range(5)] for i in range(0, K, EVERY)}
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # Untimed steps before and after the timed region (about 0.3 s each) keep the GPU under the
+    # same load while the clock sampler runs, so that a short timed region still has a clock
+    # record around it; samples taken inside the region are reported when there are enough.
+    roll = int(min(20000, max(1, 300.0 / max(warm_ms, 1e-3))))
     clocks = ClockSampler(local)
     barrier(world)
     torch.cuda.synchronize()
-    clocks.start()
+    clocks.start((t0, t1))
+    for i in range(roll):
+        step(sets[i % args.sets])
     t0.record(stream)
     for i in range(K):
         step(sets[i % args.sets], evs.get(i))
     t1.record(stream)
+    for i in range(roll):
+        step(sets[i % args.sets])
     torch.cuda.synchronize()
     barrier(world)
     clk = clocks.stop()
@@ -310,8 +416,13 @@ def run_ours(args):
     ms2 = max_over_ranks(world, e0.elapsed_time(e1), dev)
     e2e = job_value(world, OPS_STEP, K2, ms2)
 
-    peak_tflops, peak_gbs, peak_src = peaks()
-    stacks = None if args.no_stacks else run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src)
+    pk = peaks()
+    extra = {}
+    if not args.no_stacks:
+        extra.update(run_stacks(dev, stream, pk))
+    if not args.no_sweep:
+        extra["single_layer"] = run_single_layer(dev, stream, pk)
+        extra["sweep"] = run_sweep(dev, stream, pk, oracle_point=(rank == 0 and world == 1))
     achieved = (OPS_GATEUP + OPS_DOWN) / ((gemm_gu_ms + gemm_dn_ms) * 1e-3) / 1e12
     cpu = cpu_baseline(mlp, packed, args.cpu_seconds) if (rank == 0 and world == 1) else None
     if rank == 0:
@@ -322,10 +433,13 @@ def run_ours(args):
             "config": {"workload": WORKLOAD, "tokens": M, "hidden": K_IN, "mlp_hidden": HIDDEN,
                        "l2": f"{args.sets} rotating weight+activation sets (~{args.sets * 117} MB) > 129 MB L2",
                        "parallelism": f"replica per GPU x{world}"},
-            "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": round(peak_tflops, 1),
-                         "unit": "TFLOP/s", "frac": round(achieved / peak_tflops, 4), "traffic": gemm_traffic(),
+            "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": round(pk["tflops"], 1),
+                         "unit": "TFLOP/s", "frac": round(achieved / pk["tflops"], 4), "traffic": gemm_traffic(),
                          "kernel": "gemm_w4a4 (gate/up + down launches)",
-                         "peak_note": f"{peak_src} sustained bf16 x {FP8_OVER_BF16:g} (nominal E4M3/bf16 ratio)"},
+                         "peak_note": f"{pk['src']} burst bf16 x {FP8_OVER_BF16:g} (nominal E4M3/bf16 ratio); each "
+                                      "GEMM launch is timed alone by its own events",
+                         "peak_sustained": round(pk["tflops_sustained"], 1),
+                         "frac_of_sustained": round(achieved / pk["tflops_sustained"], 4)},
             "kernels_us_note": f"CUDA events around each launch on every {EVERY}th timed step",
             "kernels_us": {"rotate_quantize_x": round(rqx_ms * 1e3, 2), "gemm_gate_up": round(gemm_gu_ms * 1e3, 2),
                            "rotate_quantize_h": round(rqh_ms * 1e3, 2), "gemm_down": round(gemm_dn_ms * 1e3, 2)},
@@ -337,8 +451,7 @@ def run_ours(args):
             "clocks": clk,
             "cpu_baseline": cpu,
         }
-        if stacks:
-            line.update(stacks)
+        line.update(extra)
         print(json.dumps(line), flush=True)
     for s in sets:
         s["gu"].close()
@@ -441,11 +554,11 @@ def _w4a8_gate_up(Q, W, dev, stream, flush, peak_tflops):
     layer.close()
     tops = OPS_GATEUP / (ms * 1e-3) / 1e12
     return {"us": round(ms * 1e3, 1), "tops": round(tops, 1), "e4m3_tflops_issued": round(2 * tops, 1),
-            "frac_of_e4m3_peak": round(2 * tops / (FP8_OVER_BF16 * peak_tflops), 4),
+            "frac_of_e4m3_peak": round(2 * tops / peak_tflops, 4),
             "timing": "rotate+quantise (8-bit codes) and GEMM launches, L2 flushed before each of 20 runs"}
 
 
-def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
+def run_stacks(dev, stream, pk):
     from paper_2605_28803_gb300 import qvla as Q
     from paper_2605_28803_gb300 import stack as S
     from paper_2605_28803_gb300 import workloads as W
@@ -467,8 +580,8 @@ def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
             Q.qvla_rotated_absmax(xc, Q.F16, DIT_CAL_ROWS, w.k, w.had_block, peak, stream)
             row.append(np.float32(peak.item()))
         peaks.append(np.asarray(row, dtype=np.float32))
-    dit = _dit_stack(S, Q, W, weights, peaks, 4, dev, stream, flush, peak_gbs, peak_src)
-    dit["w4a8"] = _dit_stack(S, Q, W, weights, peaks, 8, dev, stream, flush, peak_gbs, peak_src)
+    dit = _dit_stack(S, Q, W, weights, peaks, 4, dev, stream, flush, pk["gbs"], pk["src"])
+    dit["w4a8"] = _dit_stack(S, Q, W, weights, peaks, 8, dev, stream, flush, pk["gbs"], pk["src"])
     # the paper's rotation configuration: Hadamard blocks of 64, per-step tables per 128-channel
     # group, inputs with uneven channel magnitudes
     wb = W.dit_stack_blocks(weights, 64)
@@ -482,11 +595,11 @@ def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
             Q.qvla_rotated_absmax_groups(xc, Q.F16, DIT_CAL_ROWS, w.k, w.had_block, gp, stream)
             row.append(gp.cpu().numpy())
         gpeaks.append(np.asarray(row, dtype=np.float32))
-    dit["grouped"] = _dit_stack(S, Q, W, wb, gpeaks, 4, dev, stream, flush, peak_gbs, peak_src, profile=True)
+    dit["grouped"] = _dit_stack(S, Q, W, wb, gpeaks, 4, dev, stream, flush, pk["gbs"], pk["src"], profile=True)
     dit["tables"] = ("per-step, per-layer, calibrated with qvla_rotated_absmax on a separate 16-token draw "
                      "(absmax / 7; absmax / 127 for the W4A8 variant); 'grouped': Hadamard blocks of 64 and "
                      "per-step tables per 128-channel group (qvla_rotated_absmax_groups)")
-    w4a8_gu = _w4a8_gate_up(Q, W, dev, stream, flush, peak_tflops)
+    w4a8_gu = _w4a8_gate_up(Q, W, dev, stream, flush, pk["tflops"])
 
     # ---- backbone forward at M = 816 and M = 1 (per-token scales) ----
     weights = W.backbone_stack(seed=3)
@@ -504,14 +617,14 @@ def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
         if m > 1:
             tops = st.ops / (ms * 1e-3) / 1e12
             bb["m816"] = {"us_per_forward": round(ms * 1e3, 1), "tops": round(tops, 1),
-                          "roofline": {"bound": "tensor", "achieved": round(tops, 1), "peak": round(peak_tflops, 1),
-                                       "unit": "TFLOP/s", "frac": round(tops / peak_tflops, 4)}}
+                          "roofline": {"bound": "tensor", "achieved": round(tops, 1), "peak": round(pk["tflops"], 1),
+                                       "unit": "TFLOP/s", "frac": round(tops / pk["tflops"], 4)}}
         else:
             nbytes = _algorithmic_bytes(weights, m)
             gbs = nbytes / (ms * 1e-3) / 1e9
             bb["m1"] = {"us_per_forward": round(ms * 1e3, 1),
-                        "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": round(peak_gbs, 1),
-                                     "unit": "GB/s", "frac": round(gbs / peak_gbs, 4), "bytes": nbytes}}
+                        "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": round(pk["gbs"], 1),
+                                     "unit": "GB/s", "frac": round(gbs / pk["gbs"], 4), "bytes": nbytes}}
         st.close()
         del g, st
         torch.cuda.empty_cache()
@@ -519,6 +632,174 @@ def run_stacks(dev, stream, peak_tflops, peak_gbs, peak_src):
     del scratch
     torch.cuda.empty_cache()
     return {"dit": dit, "backbone": bb, "w4a8_gate_up": w4a8_gu}
+
+
+# --------------------------------------------------------------------------------------
+# config 1 (one per-step layer) and the config-5 sweep of single linears
+# --------------------------------------------------------------------------------------
+
+def _linear_bytes(m, k, n, xb=2, yb=2):
+    """Algorithmic bytes of one fused linear: activations in, packed int4 weights, the weight
+    scales, outputs."""
+    return xb * m * k + n * k // 2 + 4 * n + yb * m * n
+
+
+def _roofline_point(ops, nbytes, sec, pk):
+    """Whichever roofline bounds a linear of this arithmetic intensity, and the fraction of it
+    reached: HBM left of the ridge (peak tensor rate / HBM bandwidth), the tensor rate right."""
+    ridge = pk["tflops"] * 1e12 / (pk["gbs"] * 1e9)
+    if ops / nbytes < ridge:
+        ach = nbytes / sec / 1e9
+        return {"bound": "hbm", "achieved": round(ach, 1), "unit": "GB/s", "frac": round(ach / pk["gbs"], 4)}
+    ach = ops / sec / 1e12
+    return {"bound": "tensor", "achieved": round(ach, 1), "unit": "TFLOP/s", "frac": round(ach / pk["tflops"], 4)}
+
+
+def run_single_layer(dev, stream, pk):
+    """The 64 x 512 x 512 per-step layer (random orthogonal SVD stand-in folded into the weights,
+    Hadamard 512, a T = 10 step table from each step's rotated absmax): one qvla_w4a4_linear
+    timed cold (L2 flushed before each call) and as one CUDA graph of the 10 steps replayed back
+    to back."""
+    from paper_2605_28803_gb300 import qvla as Q
+    from paper_2605_28803_gb300 import workloads as W
+
+    case = W.single_layer_steps(seed=0)
+    n, k = case.w.shape
+    m, steps = case.x_steps[0].shape[0], len(case.x_steps)
+    wq, ws = np.zeros((n, k // 2), np.uint8), np.zeros(n, np.float32)
+    Q.qvla_pack_weights_host(np.ascontiguousarray(case.w), Q.F32, n, k, rot=np.ascontiguousarray(case.rot),
+                             rot_block=case.rot_block, had_block=case.had_block, wq=wq, wscale=ws)
+    layer = Q.qvla_layer_create(n, k, case.had_block, Q.F16, Q.F16, wq, ws, None)
+    xs = [x.to(dev) for x in case.x_steps]
+    peak = torch.zeros(1, dtype=torch.float32, device=dev)
+    table = []
+    for t in range(steps):
+        peak.zero_()
+        Q.qvla_rotated_absmax(xs[t], Q.F16, m, k, case.had_block, peak, stream)
+        table.append(np.float32(peak.item()) / np.float32(7))
+    Q.qvla_set_step_scales(layer, np.asarray(table, np.float32))
+    y = torch.empty(m, n, dtype=torch.float16, device=dev)
+    nb = Q.qvla_linear_workspace_bytes(layer, m)
+    work = torch.empty(nb, dtype=torch.uint8, device=dev)
+    scratch = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def one(t):
+        Q.qvla_w4a4_linear(layer, xs[t], m, t, y, work, nb, stream)
+
+    for t in range(steps):
+        one(t)
+    torch.cuda.synchronize()
+    Q.qvla_check_device(stream)
+    reps = 20
+    cold_ms = sum(_time_replays(lambda t=t: one(t), reps, scratch.zero_, stream) for t in range(steps)) / steps
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for t in range(steps):
+            Q.qvla_w4a4_linear(layer, xs[t], m, t, y, work, nb, torch.cuda.current_stream())
+    g.replay()
+    torch.cuda.synchronize()
+    graph_ms = _time_replays(g.replay, reps, None, stream) / steps
+    Q.qvla_check_device(stream)
+    layer.close()
+    del g, scratch
+    torch.cuda.empty_cache()
+    nbytes, ops = _linear_bytes(m, k, n), 2 * m * n * k
+    return {"shape": f"M={m} K={k} N={n}, f16 in/out, Hadamard {case.had_block}, T={steps} step table",
+            "us_cold": round(cold_ms * 1e3, 2), "us_graph": round(graph_ms * 1e3, 2),
+            "gbs_cold": round(nbytes / (cold_ms * 1e-3) / 1e9, 1), "gbs_graph": round(nbytes / (graph_ms * 1e-3) / 1e9, 1),
+            "tops_graph": round(ops / (graph_ms * 1e-3) / 1e12, 2), "bytes": nbytes, "ops": ops,
+            "frac_hbm_graph": round(nbytes / (graph_ms * 1e-3) / 1e9 / pk["gbs"], 4),
+            "timing": "qvla_w4a4_linear (2 launches); cold: L2 flushed before each of 20 calls per step; "
+                      "graph: the 10 steps captured once, replayed back to back, time / 10"}
+
+
+SWEEP_M = (1, 16, 50, 256, 816, 3200, 8192)
+SWEEP_KN = ((1024, 1024), (1024, 4096), (2048, 2048), (2048, 16384), (16384, 2048))
+
+
+def run_sweep(dev, stream, pk, oracle_point=True):
+    """The single-linear sweep: qvla_w4a4_linear at M in SWEEP_M x (K, N) in SWEEP_KN, f16 in and
+    out, per-token scales, Hadamard K (2048 blocks at K = 16384).  Each point: 10 calls, L2
+    flushed before each, CUDA events around the rotate + quantise and the GEMM launches.  The
+    weights are uniform random code bytes (the time of a linear does not depend on its values);
+    the activations are drawn on the device (N(0,1), 0.5% channels x20)."""
+    from paper_2605_28803_gb300 import qvla as Q
+    from paper_2605_28803_gb300 import workloads as W
+
+    scratch = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    mmax = max(SWEEP_M)
+    points = []
+    for kn_i, (k, n) in enumerate(SWEEP_KN):
+        had = k if k <= 4096 else 2048
+        rng = np.random.default_rng(500 + kn_i)
+        packed = rng.integers(0, 256, (n, k // 2), dtype=np.uint8)
+        ws = (rng.uniform(0.8, 1.2, n) * 0.5 / np.sqrt(k)).astype(np.float32)
+        layer = Q.qvla_layer_create(n, k, had, Q.F16, Q.F16, packed, ws, None)
+        x = W.sweep_input_device(mmax, k, seed=600 + kn_i, device=dev, dtype="f16")
+        y = torch.empty(mmax, n, dtype=torch.float16, device=dev)
+        nb = Q.qvla_linear_workspace_bytes(layer, mmax)
+        work = torch.empty(nb, dtype=torch.uint8, device=dev)
+        for m in SWEEP_M:
+            xm, ym = x[:m], y[:m]
+
+            def call(ev=None):
+                if ev:
+                    ev[0].record(stream)
+                Q.qvla_linear_quantize(layer, xm, m, -1, work, nb, stream)
+                if ev:
+                    ev[1].record(stream)
+                Q.qvla_linear_gemm(layer, work, nb, m, ym, stream)
+                if ev:
+                    ev[2].record(stream)
+
+            for _ in range(3):
+                call()
+            torch.cuda.synchronize()
+            evs = []
+            for _ in range(10):
+                scratch.zero_()
+                e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+                call(e)
+                evs.append(e)
+            torch.cuda.synchronize()
+            t_all = statistics.median(e[0].elapsed_time(e[2]) for e in evs) * 1e-3
+            t_rq = statistics.median(e[0].elapsed_time(e[1]) for e in evs) * 1e-3
+            t_gemm = statistics.median(e[1].elapsed_time(e[2]) for e in evs) * 1e-3
+            ops, nbytes = 2 * m * n * k, _linear_bytes(m, k, n)
+            pt = {"M": m, "K": k, "N": n, "us": round(t_all * 1e6, 2), "us_rotate_quantize": round(t_rq * 1e6, 2),
+                  "us_gemm": round(t_gemm * 1e6, 2), "tops": round(ops / t_all / 1e12, 2),
+                  "gbs": round(nbytes / t_all / 1e9, 1)}
+            pt["roofline"] = _roofline_point(ops, nbytes, t_all, pk)
+            points.append(pt)
+        Q.qvla_check_device(stream)
+        layer.close()
+        del x, y, work
+        torch.cuda.empty_cache()
+    del scratch
+    torch.cuda.empty_cache()
+    out = {"points": points,
+           "timing": "median of 10 calls of qvla_w4a4_linear's two halves, L2 flushed (256 MB write) before each; "
+                     "bytes = 2MK + NK/2 + 4N + 2MN; roofline = HBM left of the ridge, burst E4M3 right of it",
+           "ridge_ops_per_byte": round(pk["tflops"] * 1e12 / (pk["gbs"] * 1e9), 1)}
+    if oracle_point:
+        out["oracle_point"] = _oracle_sweep_point()
+    return out
+
+
+def _oracle_sweep_point(m=256, k=2048, n=2048):
+    """The oracle's host time for one sweep point (K, N) = (2048, 2048), M = 256: rotate,
+    quantise, integer GEMM and dequantise in numpy float64 (the offline weight pack not timed)."""
+    from oracle import qvla_oracle as O
+    from paper_2605_28803_gb300 import workloads as W
+
+    case = W.sweep_linear(m, k, n, seed=4, xdtype="f16", ydtype="f16")
+    _, ws, codes = O.pack_weights(case.w.astype(np.float64), case.had_block)
+    x64 = case.x.double().numpy()
+    t0 = time.perf_counter()
+    O.w4a4_linear(x64, codes, ws, case.had_block, out_fmt="f16")
+    el = time.perf_counter() - t0
+    return {"M": m, "K": k, "N": n, "seconds": round(el, 3), "tops": round(2 * m * n * k / el / 1e12, 6),
+            "cores": cpu_cores(), "kind": "oracle"}
 
 
 # --------------------------------------------------------------------------------------

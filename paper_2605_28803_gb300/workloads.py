@@ -149,6 +149,19 @@ def sweep_linear(m: int, k: int, n: int, seed: int = 4, outlier_frac: float = 0.
     return LinearCase(as_dtype(x, xdtype), w, bias, had_block, xdtype, ydtype)
 
 
+def sweep_input_device(m: int, k: int, seed: int, device, dtype: str = "f16", outlier_frac: float = 0.005,
+                       outlier_factor: float = 20.0) -> torch.Tensor:
+    """Sweep activations drawn on the device with torch's seeded generator (the largest sweep
+    points hold 134 M values, seconds of host drawing): N(0,1) [m, k] with round(0.5% K)
+    channels x20.  Draw order: X, then the outlier channels."""
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    x = torch.randn(m, k, generator=g, device=device, dtype=torch.float32)
+    idx = torch.randperm(k, generator=g, device=device)[:max(1, int(round(outlier_frac * k)))]
+    x[:, idx] *= outlier_factor
+    return x.to(_TORCH_DTYPES[dtype])
+
+
 def dit_input_std(t: int, steps: int = 10, start: float = 4.0, end: float = 0.5) -> float:
     """Per-step input magnitude of the DiT head: geometric drift from 4.0 at t = 0 to 0.5
     at t = T-1, i.e. sigma_t = 4 (1/8)^(t / 9) for T = 10."""

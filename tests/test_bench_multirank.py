@@ -68,3 +68,17 @@ def test_reference_arm_under_torchrun_prints_once_from_rank_zero():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["steps"] == 1
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_clock_record_prefers_samples_inside_the_timed_region():
+    sys.path.insert(0, ROOT)
+    import bench
+
+    rows = [(1900.0, 2070.0, 900.0, ["sw_power_cap"], False)] * 5 + [(2070.0, 2070.0, 800.0, [], True)] * 3
+    c = bench.ClockSampler.summarize(rows, "test")
+    assert c["sm_mhz"] == 2070.0 and c["samples_in_timed_region"] == 3 and c["reasons"] == []
+    assert c["window"] == "the timed region"
+    # fewer than three samples inside: the bracketing window, with its reasons
+    c = bench.ClockSampler.summarize(rows[:6], "test")
+    assert c["sm_mhz"] == 1900.0 and c["reasons"] == ["sw_power_cap"] and c["samples"] == 6
+    assert bench.ClockSampler.summarize([], "test") is None
