@@ -264,6 +264,22 @@ size_t qvla_linear_workspace_bytes(const qvla_layer* layer, int M);
 qvla_status qvla_w4a4_linear(const qvla_layer* layer, const void* x, int M, int step, void* y,
                              void* workspace, size_t workspace_bytes, void* stream);
 
+/* The one-launch linear for a small batch with a per-step scale: the rotation, the quantiser, the
+ * integer GEMM and the epilogue of qvla_w4a4_linear (same arithmetic, same results) in a single
+ * kernel -- the DiT head's case (Sec. 4.2, Eq. 6: the scale is the step's table entry, so no
+ * reduction along a row precedes the quantiser).  The CTAs that split the reduction over K
+ * rotate and quantise the token rows among themselves and exchange the codes in shared memory;
+ * nothing goes through a workspace.  Every CTA of a cluster rotates whole token rows, so each
+ * weight tile's cluster repeats the rotation of all M rows: on GB300 this takes longer than the
+ * two launches of qvla_w4a4_linear at every DiT shape measured except K = 512 at M = 1, and
+ * qvla_w4a4_linear does not use it.  x device [M][K] (f16 or bf16), y device out [M][N], step in
+ * [0, T).
+ * QVLA_ERR_UNSUPPORTED (nothing enqueued) where it does not apply: step == -1, M > 128, K outside
+ * [512, 4096] or not a multiple of the task width (512 channels up to K = 512, 1024 up to 1024,
+ * 2048 beyond), activation and output dtypes that differ or are f32, gated layers, per-group
+ * tables, an online P.U, or no split of K whose tiles fit the kernel's shared memory. */
+qvla_status qvla_w4a4_linear_fused(const qvla_layer* layer, const void* x, int M, int step, void* y, void* stream);
+
 /* The two halves of qvla_w4a4_linear, for callers that schedule them separately (for example to
  * time them, or to overlap one layer's GEMM with the next layer's rotation on another stream).
  * qvla_linear_quantize rotates and quantises x into `workspace` (as qvla_rotate_quantize, step

@@ -701,6 +701,62 @@ qvla_status qvla_linear_gemm(const qvla_layer* L, const void* workspace, size_t 
   return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream);
 }
 
+namespace {
+// The one-launch linear (fused rotate + quantise prologue in the GEMM) where the layer and batch
+// allow it: a per-step scale (one per tensor), no online P.U, not gated, f16/bf16 activations,
+// M <= 128.  *launched tells whether it was enqueued.
+qvla_status try_fused(const qvla_layer* L, const void* x, int M, const float* step_scale, void* y, void* stream,
+                      bool* launched) {
+  *launched = false;
+  if (!step_scale || L->grouped || L->rblock || L->gated || M > 128 || (L->xdt != QVLA_F16 && L->xdt != QVLA_BF16))
+    return QVLA_OK;
+  qvla::GemmArgs a;
+  a.xq = nullptr;
+  a.x_bytes = 3;
+  a.xscale = step_scale;
+  a.xsum = nullptr;
+  a.wq = L->wq;
+  a.wscale = L->wscale;
+  a.wcorr = L->wcorr;
+  a.bias = L->bias;
+  a.y = y;
+  a.ydt = L->ydt;
+  a.acc = nullptr;
+  a.M = M;
+  a.N = L->N;
+  a.K = L->K;
+  a.gated = 0;
+  a.x = x;
+  a.xdt = L->xdt;
+  a.log_b = L->log_b;
+  a.inv_sqrt_b = static_cast<float>(1.0 / std::sqrt(static_cast<double>(L->had_block)));
+  a.num_sms = num_sms(L->device);
+  a.stream = static_cast<cudaStream_t>(stream);
+  QVLA_CUDA(qvla::launch_gemm_fused(a, launched), "fused linear launch");
+  return QVLA_OK;
+}
+}  // namespace
+
+qvla_status qvla_w4a4_linear_fused(const qvla_layer* L, const void* x, int M, int step, void* y, void* stream) {
+  g_last_error.clear();
+  if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
+  if (qvla_status s = check_rows(M)) return s;
+  if (step < 0) return fail(QVLA_ERR_UNSUPPORTED, "the one-launch linear takes a per-step scale (step >= 0)");
+  const float* ss = nullptr;
+  if (qvla_status s = resolve_step(L, step, &ss)) return s;
+  if (M == 0) return QVLA_OK;
+  if (!x || !y) return fail(QVLA_ERR_INVALID_ARG, "x and y must not be NULL");
+  if (!aligned16(x) || !aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "x and y must be 16-byte aligned");
+  if (qvla_status s = check_layer_device(L)) return s;
+  bool launched = false;
+  if (qvla_status s = try_fused(L, x, M, ss, y, stream, &launched)) return s;
+  if (!launched)
+    return fail(QVLA_ERR_UNSUPPORTED,
+                "the one-launch linear does not take this layer or batch (M=%d, K=%d, N=%d): use qvla_w4a4_linear", M,
+                L->K, L->N);
+  return QVLA_OK;
+}
+
 qvla_status qvla_w4a4_linear(const qvla_layer* L, const void* x, int M, int step, void* y, void* workspace,
                              size_t workspace_bytes, void* stream) {
   g_last_error.clear();
@@ -848,9 +904,10 @@ qvla_status qvla_w4a4_linear_noalloc(const qvla_layer* L, const void* x, int M, 
 
 qvla_status qvla_check_device(void* stream) {
   g_last_error.clear();
-  unsigned int word = 0;
+  unsigned int word = 0, word_fused = 0;
   QVLA_CUDA(qvla::read_and_clear_error_word(&word, static_cast<cudaStream_t>(stream)), "device check");
-  if (word & 1u) return fail(QVLA_ERR_TIMEOUT, "a kernel wait ran out of its time limit");
+  QVLA_CUDA(qvla::read_and_clear_error_word_fused(&word_fused, static_cast<cudaStream_t>(stream)), "device check");
+  if ((word | word_fused) & 1u) return fail(QVLA_ERR_TIMEOUT, "a kernel wait ran out of its time limit");
   return QVLA_OK;
 }
 

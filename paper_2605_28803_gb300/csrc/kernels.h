@@ -71,12 +71,25 @@ struct GemmArgs {
   const int32_t* xgsum = nullptr;
   const float* wgcorr = nullptr;
   int group = 0;
+  // the fused one-launch linear (launch_gemm_fused): raw activations x [M][K] of dtype xdt
+  // (0 f16, 1 bf16) with Hadamard block 2^log_b; xscale then points at the step's one scale
+  const void* x = nullptr;
+  int xdt = 0;
+  int log_b = 0;
+  float inv_sqrt_b = 1.0f;
   int num_sms;
   cudaStream_t stream;
 };
 cudaError_t launch_gemm_w4a4(const GemmArgs& a);
 
-// Read and clear the device-side error word of the kernels that wait (gemm.cu).
+// The one-launch linear for a small batch with a per-step scale (gemm_fused.cu): the weight-major
+// split-K GEMM whose CTAs rotate and quantise the activations themselves.  *launched is false
+// (and nothing was enqueued) when the shape is outside what it takes: M > 128, gated or grouped
+// layers, K beyond 4096, or no split of K that fits its shared-memory tiles.
+cudaError_t launch_gemm_fused(const GemmArgs& a, bool* launched);
+
+// Read and clear the device-side error words of the kernels that wait (gemm.cu, gemm_fused.cu).
 cudaError_t read_and_clear_error_word(unsigned int* out, cudaStream_t stream);
+cudaError_t read_and_clear_error_word_fused(unsigned int* out, cudaStream_t stream);
 
 }  // namespace qvla

@@ -49,6 +49,7 @@ SIGNATURES = {
     "qvla_linear_quantize": (_I, [_P, _P, _I, _I, _P, _S, _P]),
     "qvla_linear_gemm": (_I, [_P, _P, _S, _I, _P, _P]),
     "qvla_w4a4_linear_noalloc": (_I, [_P, _P, _I, _I, _P, _P]),
+    "qvla_w4a4_linear_fused": (_I, [_P, _P, _I, _I, _P, _P]),
     "qvla_rotate_quantize_rows_a8": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
     "qvla_w4a8_workspace_bytes": (_S, [_P, _I]),
     "qvla_w4a8_linear": (_I, [_P, _P, _I, _I, _P, _P, _S, _P]),
@@ -258,6 +259,11 @@ def qvla_linear_gemm(layer: Layer, workspace, workspace_bytes: int, M: int, y, s
 
 
 NOALLOC_SCRATCH_BYTES = 8 << 20
+
+
+def qvla_w4a4_linear_fused(layer: Layer, x, M: int, step: int, y, stream=None) -> None:
+    """The one-launch linear (small batch, per-step scale); QvlaError status 2 where it does not apply."""
+    _check(_lib.qvla_w4a4_linear_fused(layer.handle, _ptr(x), M, step, _ptr(y), _stream(stream)))
 
 
 def qvla_w4a4_linear_noalloc(layer: Layer, x, M: int, step: int, y, stream=None) -> None:

@@ -51,8 +51,8 @@ def test_dit_stack_every_linear_at_three_steps():
                                     out_fmt="f16")
                 clamped += int(np.count_nonzero(np.abs(ref["y_rot"]) > 7.5 * float(tables[i][t])))
                 got = st.y[i].double().cpu().numpy()
-                G.assert_output_close(got, ref["y"], "f16")
-                assert np.mean(got == ref["y"]) > 0.98, w.name
+                adj = G.assert_linear_close_modulo_ties(got, ref, w.codes, w.wscale, w.bias, "f16")
+                assert np.mean(got == adj) > 0.98, w.name
     finally:
         st.close()
     assert clamped > 0, "the evaluation draw never exceeded the calibrated range"
