@@ -12,6 +12,7 @@
 #include <vector>
 
 #include "../../include/qvla.h"
+#include "../../include/qvla_debug.h"
 #include "kernels.h"
 #include "pack.h"
 
@@ -900,6 +901,15 @@ qvla_status qvla_w4a4_linear_noalloc(const qvla_layer* L, const void* x, int M, 
   void* scratch = nullptr;
   if (qvla_status s = noalloc_scratch(&scratch)) return s;
   return qvla_w4a4_linear(L, x, M, step, y, scratch, QVLA_NOALLOC_SCRATCH_BYTES, stream);
+}
+
+qvla_status qvla_debug_set_hooks(unsigned long long wait_limit_ns, int hold_gemm_loads) {
+  g_last_error.clear();
+  const unsigned long long limit = wait_limit_ns ? wait_limit_ns : 2000000000ull;
+  const int hold = hold_gemm_loads ? 1 : 0;
+  QVLA_CUDA(qvla::set_debug_hooks_gemm(limit, hold), "test hooks (gemm)");
+  QVLA_CUDA(qvla::set_debug_hooks_fused(limit, hold), "test hooks (fused)");
+  return QVLA_OK;
 }
 
 qvla_status qvla_check_device(void* stream) {

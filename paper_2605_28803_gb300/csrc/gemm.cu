@@ -94,6 +94,10 @@ cudaError_t launch_gemm_w4a4(const GemmArgs& a) {
   return a.ydt == 0 ? launch_out<0, __half>(a) : launch_out<0, __nv_bfloat16>(a);
 }
 
+cudaError_t set_debug_hooks_gemm(unsigned long long wait_limit_ns, int hold_loads) {
+  return set_debug_hooks(wait_limit_ns, hold_loads);
+}
+
 cudaError_t read_and_clear_error_word(unsigned int* out, cudaStream_t stream) {
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return e;

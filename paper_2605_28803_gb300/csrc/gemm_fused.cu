@@ -35,6 +35,10 @@ cudaError_t launch_gemm_fused(const GemmArgs& a, bool* launched) {
   return e;
 }
 
+cudaError_t set_debug_hooks_fused(unsigned long long wait_limit_ns, int hold_loads) {
+  return set_debug_hooks(wait_limit_ns, hold_loads);
+}
+
 cudaError_t read_and_clear_error_word_fused(unsigned int* out, cudaStream_t stream) {
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return e;

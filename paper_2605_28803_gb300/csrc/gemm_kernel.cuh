@@ -53,6 +53,10 @@
 namespace qvla {
 namespace {
 
+// Test hook (qvla_debug_hold_gemm_loads): while set, the load warp of a GEMM issues no copy at all,
+// so every wait on those copies runs out (see qvla_debug.h).  Per translation unit.
+static __device__ int g_debug_hold_loads;
+
 constexpr int kBM = 128;        // MMA M (rows of the MMA A operand)
 constexpr int kBK = 128;        // codes per k-block (one 128-byte swizzle row of E4M3)
 constexpr int kEpiWarps = 4;
@@ -475,10 +479,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     if (threadIdx.x == 0)
       mbar_arrive_expect_tx(smem_u32(&bar_xready), static_cast<uint32_t>(p.M * (kb1 - kb0) * kBK));
   }
+  // split-K: the token columns of this cluster's tile that hold tokens (only those are exchanged)
+  const int split_cols = kSwap ? max(0, min(kBN, p.rows_b - static_cast<int>(QVLA_UNIT0 / static_cast<unsigned>(tiles_a)) * kBN))
+                               : kBN;
   if (kSwap && splits > 1) {
     // split-K: this CTA receives one slice of its rows from every CTA of the cluster; the
     // cluster barrier completed before the first send guarantees every receiver's barrier exists
-    if (threadIdx.x == 0) mbar_arrive_expect_tx(smem_u32(&bar_recv), static_cast<uint32_t>(kBM * kBN * 4));
+    if (threadIdx.x == 0) mbar_arrive_expect_tx(smem_u32(&bar_recv), static_cast<uint32_t>(kBM * split_cols * 4));
     if constexpr (kFused) {
       cluster_sync();  // the prologue sends early: every barrier of the cluster exists from here on
     } else {
@@ -536,9 +543,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       // only, which no earlier kernel writes, so the first stages are requested before waiting
       // for the previous kernel (a small batch's GEMM is mostly this latency).
       int pre = 0;
+      const bool hold = *const_cast<volatile int*>(&g_debug_hold_loads) != 0;  // test hook: issue nothing
       if constexpr ((kXBytes || kFused) && kSwap) {
         const int unit0 = static_cast<int>(QVLA_UNIT0);
-        if (unit0 < ntiles) {
+        if (unit0 < ntiles && !hold) {
           const int ta = unit0 % tiles_a;
           pre = min(C::kStages, kb1 - kb0);
           for (int i = 0; i < pre; ++i) {
@@ -550,7 +558,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       }
       griddep_wait();
       int it = 0;
-      bool ok = true;
+      bool ok = !hold;
       for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS) {
         const int ta = tile % tiles_a, tb = tile / tiles_a;
         for (int kb = kb0; kb < kb1; ++kb, ++it) {
@@ -1119,12 +1127,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
         const uint32_t rbar = mapa_shared(smem_u32(&bar_recv), static_cast<uint32_t>(owner));
         const uint32_t rdst = mapa_shared(recv0, static_cast<uint32_t>(owner)) +
                               static_cast<uint32_t>((static_cast<int>(krank) * kBN * R + (row - owner * R)) * 4);
-        for (int col = static_cast<int>(threadIdx.x) / (kBM / 4); col < kBN; col += kThreads / (kBM / 4))
+        for (int col = static_cast<int>(threadIdx.x) / (kBM / 4); col < split_cols; col += kThreads / (kBM / 4))
           st_async_v4(rdst + static_cast<uint32_t>(col * R * 4), *reinterpret_cast<const float4*>(part + col * kBM + row), rbar);
       }
       const int R4 = R / 4;
       const int unit0 = static_cast<int>(QVLA_UNIT0);
-      const int total = unit0 < ntiles && !s_epi_abort ? R4 * kBN : 0;
+      const int total = unit0 < ntiles && !s_epi_abort ? R4 * split_cols : 0;
       const int ta = unit0 % tiles_a, tb = unit0 / tiles_a;
       auto coords = [&](int e, int& n, int& m, int& row, int& col) {
         row = (e % R4) * 4;  // within this CTA's R rows
@@ -1443,6 +1451,15 @@ cudaError_t launch_cfg(const GemmArgs& a) {
   e = cudaLaunchKernelEx(&cfg, kern, ta, tb, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+// Test hooks of the kernels instantiated in the including translation unit.
+inline cudaError_t set_debug_hooks(unsigned long long wait_limit_ns, int hold_loads) {
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return e;
+  e = cudaMemcpyToSymbol(g_wait_limit_ns, &wait_limit_ns, sizeof(wait_limit_ns));
+  if (e != cudaSuccess) return e;
+  return cudaMemcpyToSymbol(g_debug_hold_loads, &hold_loads, sizeof(hold_loads));
 }
 
 }  // namespace

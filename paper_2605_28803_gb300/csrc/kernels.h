@@ -92,4 +92,9 @@ cudaError_t launch_gemm_fused(const GemmArgs& a, bool* launched);
 cudaError_t read_and_clear_error_word(unsigned int* out, cudaStream_t stream);
 cudaError_t read_and_clear_error_word_fused(unsigned int* out, cudaStream_t stream);
 
+// Test hooks (qvla_debug.h): the wait limit of the bounded waits and whether GEMM load warps hold
+// back every copy, for the kernels of gemm.cu and of gemm_fused.cu.  Synchronise the device first.
+cudaError_t set_debug_hooks_gemm(unsigned long long wait_limit_ns, int hold_loads);
+cudaError_t set_debug_hooks_fused(unsigned long long wait_limit_ns, int hold_loads);
+
 }  // namespace qvla

@@ -12,8 +12,10 @@ static __device__ unsigned int g_error_word;
 
 constexpr unsigned int kErrTimeout = 1u;
 // A wait gives up after this many nanoseconds of the global timer (a healthy wait in these
-// kernels lasts microseconds).
+// kernels lasts microseconds).  g_wait_limit_ns holds the limit in force (per translation unit,
+// like the error word); only a test hook lowers it.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+static __device__ unsigned long long g_wait_limit_ns = kWaitLimitNs;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -68,9 +70,10 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parit
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer();
+  const unsigned long long limit = *const_cast<volatile unsigned long long*>(&g_wait_limit_ns);
   for (;;) {
     if (mbar_try_wait_sleep(bar, parity)) return true;
-    if (globaltimer() - t0 > kWaitLimitNs) {
+    if (globaltimer() - t0 > limit) {
       atomicOr(&g_error_word, kErrTimeout);
       return false;
     }
@@ -177,9 +180,10 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t par
 __device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity) {
   if (mbar_try_wait_cluster(bar, parity)) return true;
   const unsigned long long t0 = globaltimer();
+  const unsigned long long limit = *const_cast<volatile unsigned long long*>(&g_wait_limit_ns);
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
-    if ((i & 255u) == 0 && globaltimer() - t0 > kWaitLimitNs) {
+    if ((i & 255u) == 0 && globaltimer() - t0 > limit) {
       atomicOr(&g_error_word, kErrTimeout);
       return false;
     }

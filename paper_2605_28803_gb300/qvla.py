@@ -21,7 +21,7 @@ DTYPE_CODES = {"f16": F16, "bf16": BF16, "f32": F32}
 STATUS = {0: "QVLA_OK", 1: "QVLA_ERR_INVALID_ARG", 2: "QVLA_ERR_UNSUPPORTED", 3: "QVLA_ERR_CUDA",
           4: "QVLA_ERR_OOM", 5: "QVLA_ERR_STEP_RANGE", 6: "QVLA_ERR_TIMEOUT"}
 
-# every symbol include/qvla.h declares, with (restype, argtypes)
+# every symbol include/*.h declares, with (restype, argtypes)
 _P, _I, _S, _D = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_double
 SIGNATURES = {
     "qvla_last_error": (ctypes.c_char_p, []),
@@ -55,6 +55,7 @@ SIGNATURES = {
     "qvla_w4a8_linear": (_I, [_P, _P, _I, _I, _P, _P, _S, _P]),
     "qvla_gemm_w4a8": (_I, [_P, _P, _P, _I, _P, _P, _P, _S, _P]),
     "qvla_check_device": (_I, [_P]),
+    "qvla_debug_set_hooks": (_I, [ctypes.c_ulonglong, _I]),
 }
 
 
@@ -294,3 +295,9 @@ def qvla_gemm_w4a8(layer: Layer, xq, xscale, M: int, y, acc, workspace, workspac
 
 def qvla_check_device(stream=None) -> None:
     _check(_lib.qvla_check_device(_stream(stream)))
+
+
+def qvla_debug_set_hooks(wait_limit_ns: int = 0, hold_gemm_loads: bool = False) -> None:
+    """Test hooks (include/qvla_debug.h): the device wait limit (0 = default) and whether GEMM
+    load warps hold back every copy."""
+    _check(_lib.qvla_debug_set_hooks(int(wait_limit_ns), 1 if hold_gemm_loads else 0))

@@ -3,6 +3,7 @@ rejects bad arguments before touching a GPU, and its host-only weight pack (fold
 int4 RTN + nibble packing) matches the oracle bit for bit."""
 
 import ctypes
+import glob
 import os
 import re
 
@@ -17,9 +18,11 @@ from tests.conftest import ROOT
 
 
 def header_symbols():
-    src = open(os.path.join(ROOT, "include", "qvla.h")).read()
-    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"\b(qvla_[a-z0-9_]+)\s*\(", src)))
+    names = set()
+    for h in sorted(glob.glob(os.path.join(ROOT, "include", "*.h"))):
+        src = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names |= set(re.findall(r"\b(qvla_[a-z0-9_]+)\s*\(", src))
+    return sorted(names)
 
 
 def test_every_declared_symbol_is_exported():

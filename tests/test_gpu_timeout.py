@@ -1,0 +1,50 @@
+"""The device-side failure path: a bounded wait that runs out.
+
+A test hook (include/qvla_debug.h) makes the GEMM's load warp issue no copy and shortens the wait
+limit to 20 ms, so the converters' waits for the staged tiles, the MMA thread's wait for the
+expanded tiles and the epilogue's wait for the accumulator all run out.  The kernel must record
+QVLA_ERR_TIMEOUT, issue no MMA, leave the output untouched and return; qvla_check_device reports
+it once and clears it, and the next launch is bit-exact.  The held kernel has no copy, MMA or
+asynchronous store outstanding when it returns (it is the token-major single-CTA form: no cluster
+exchange), so nothing faults or hangs."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import qvla_oracle as O
+from paper_2605_28803_gb300 import qvla as Q
+from tests import gpu_helpers as G
+
+pytestmark = pytest.mark.gpu
+
+
+def test_a_wait_that_runs_out_reports_timeout_and_the_next_launch_is_clean():
+    rng = np.random.default_rng(61)
+    M, K, N = 256, 512, 256
+    wcodes = rng.integers(-7, 8, (N, K)).astype(np.int8)
+    layer = G.make_layer(O.pack_int4(wcodes), np.full(N, 0.01, np.float32), 512, "f16", "f16")
+    xcodes = rng.integers(-7, 8, (M, K)).astype(np.int8)
+    xq, xs = O.pack_int4(xcodes), np.full(M, 0.02, np.float32)
+    xsum = xcodes.astype(np.int64).sum(1)
+    y0, acc0 = G.gemm(layer, xq, xs, xsum)
+    assert np.array_equal(acc0, O.int_gemm(xcodes, wcodes))
+
+    xqg = torch.from_numpy(xq).to(G.DEV)
+    xsg = torch.from_numpy(xs).to(G.DEV)
+    xsumg = torch.from_numpy(xsum.astype(np.int32)).to(G.DEV)
+    y = torch.full((M, N), float("nan"), dtype=torch.float16, device=G.DEV)
+    Q.qvla_check_device(G.stream())
+    Q.qvla_debug_set_hooks(20_000_000, True)
+    try:
+        Q.qvla_gemm_w4a4(layer, xqg, xsg, xsumg, M, y, None, G.stream())
+        with pytest.raises(Q.QvlaError) as e:
+            Q.qvla_check_device(G.stream())
+        assert e.value.status == 6
+        assert torch.isnan(y).all().item()  # nothing was written
+    finally:
+        Q.qvla_debug_set_hooks(0, False)
+    Q.qvla_check_device(G.stream())  # the error word was cleared by the first check
+    y1, acc1 = G.gemm(layer, xq, xs, xsum)
+    assert np.array_equal(acc1, acc0) and np.array_equal(y1, y0)
+    layer.close()
