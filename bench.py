@@ -63,6 +63,8 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="CPU-baseline sample budget")
     ap.add_argument("--no-stacks", action="store_true", help="skip the DiT and backbone stack legs")
     ap.add_argument("--no-sweep", action="store_true", help="skip the single-layer and sweep legs")
+    ap.add_argument("--sweep-points", default=None,
+                    help="only time these sweep points, 'M,K,N;M,K,N' (a short run for profiling); prints their line")
     return ap.parse_args()
 
 
@@ -253,6 +255,14 @@ class ClockSampler:
                 "how": how}
 
 
+def gemm_source_hash():
+    """sha256 over the GEMM kernel's sources (the kernel template and its dispatch)."""
+    h = hashlib.sha256()
+    for f in ("gemm_kernel.cuh", "gemm.cu", "ptx.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2605_28803_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()
+
+
 def gemm_traffic():
     """dram bytes per launch of the GEMM kernel from the committed ncu summary, or None if the
     kernel source changed since the counters were taken."""
@@ -260,8 +270,7 @@ def gemm_traffic():
     if not os.path.exists(p):
         return None
     d = json.load(open(p))
-    src = open(os.path.join(ROOT, "paper_2605_28803_gb300", "csrc", "gemm.cu"), "rb").read()
-    if hashlib.sha256(src).hexdigest() != d.get("gemm_cu_sha256"):
+    if gemm_source_hash() != d.get("gemm_source_sha256"):
         return None
     return d.get("dram_bytes_per_step")
 
@@ -717,7 +726,7 @@ SWEEP_M = (1, 16, 50, 256, 816, 3200, 8192)
 SWEEP_KN = ((1024, 1024), (1024, 4096), (2048, 2048), (2048, 16384), (16384, 2048))
 
 
-def run_sweep(dev, stream, pk, oracle_point=True):
+def run_sweep(dev, stream, pk, oracle_point=True, points_only=None):
     """The single-linear sweep: qvla_w4a4_linear at M in SWEEP_M x (K, N) in SWEEP_KN, f16 in and
     out, per-token scales, Hadamard K (2048 blocks at K = 16384).  Each point: 10 calls, L2
     flushed before each, CUDA events around the rotate + quantise and the GEMM launches.  The
@@ -729,17 +738,20 @@ def run_sweep(dev, stream, pk, oracle_point=True):
     scratch = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     mmax = max(SWEEP_M)
     points = []
-    for kn_i, (k, n) in enumerate(SWEEP_KN):
+    kn_list = SWEEP_KN if points_only is None else sorted({(k, n) for _, k, n in points_only})
+    for kn_i, (k, n) in enumerate(kn_list):
         had = k if k <= 4096 else 2048
         rng = np.random.default_rng(500 + kn_i)
         packed = rng.integers(0, 256, (n, k // 2), dtype=np.uint8)
         ws = (rng.uniform(0.8, 1.2, n) * 0.5 / np.sqrt(k)).astype(np.float32)
         layer = Q.qvla_layer_create(n, k, had, Q.F16, Q.F16, packed, ws, None)
-        x = W.sweep_input_device(mmax, k, seed=600 + kn_i, device=dev, dtype="f16")
-        y = torch.empty(mmax, n, dtype=torch.float16, device=dev)
-        nb = Q.qvla_linear_workspace_bytes(layer, mmax)
+        x = W.sweep_input_device(mmax if points_only is None else max(m for m, _, _ in points_only), k,
+                                 seed=600 + kn_i, device=dev, dtype="f16")
+        y = torch.empty(x.shape[0], n, dtype=torch.float16, device=dev)
+        nb = Q.qvla_linear_workspace_bytes(layer, x.shape[0])
         work = torch.empty(nb, dtype=torch.uint8, device=dev)
-        for m in SWEEP_M:
+        ms = SWEEP_M if points_only is None else sorted({m for m, kk, nn in points_only if (kk, nn) == (k, n)})
+        for m in ms:
             xm, ym = x[:m], y[:m]
 
             def call(ev=None):
@@ -891,10 +903,22 @@ def run_reference(args, budget_s: float = 90.0):
     print(json.dumps(line), flush=True)
 
 
+def run_points(args):
+    """Only the named sweep points (3 untimed and 10 timed calls each): a short run whose kernel
+    launches a profiler can pick out."""
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    pts = [tuple(int(v) for v in p.split(",")) for p in args.sweep_points.split(";") if p.strip()]
+    out = run_sweep(dev, torch.cuda.current_stream(), peaks(), oracle_point=False, points_only=pts)
+    print(json.dumps({"sweep_points": out["points"]}), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif args.sweep_points:
+        run_points(args)
     else:
         run_ours(args)
 
