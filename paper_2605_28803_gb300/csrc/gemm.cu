@@ -88,6 +88,11 @@ cudaError_t launch_out(const GemmArgs& a) {
 
 cudaError_t launch_gemm_w4a4(const GemmArgs& a) {
   if (a.M == 0) return cudaSuccess;
+  {  // one to four tokens: the weight stream decides, so the CUDA-core GEMV takes it
+    bool launched = false;
+    const cudaError_t e = launch_gemv_w4a4(a, &launched);
+    if (e != cudaSuccess || launched) return e;
+  }
   if (a.gscale) return a.ydt == 0 ? launch_grouped<__half>(a) : launch_grouped<__nv_bfloat16>(a);
   if (a.x_bytes == 2) return a.ydt == 0 ? launch_out<2, __half>(a) : launch_out<2, __nv_bfloat16>(a);
   if (a.x_bytes == 1) return a.ydt == 0 ? launch_out<1, __half>(a) : launch_out<1, __nv_bfloat16>(a);

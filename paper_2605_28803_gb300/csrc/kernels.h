@@ -88,6 +88,13 @@ cudaError_t launch_gemm_w4a4(const GemmArgs& a);
 // layers, K beyond 4096, or no split of K that fits its shared-memory tiles.
 cudaError_t launch_gemm_fused(const GemmArgs& a, bool* launched);
 
+// Decode-sized batches (gemv.cu): the integer product and epilogue on the CUDA cores for
+// M <= kGemvMaxM tokens, with activations as operand bytes (x_bytes 1) or packed codes (0), gated
+// or not, one scale per token or per step (no per-group tables).  *launched is false (nothing
+// enqueued) outside that range.  The outputs are those of launch_gemm_w4a4, bit for bit.
+constexpr int kGemvMaxM = 4;
+cudaError_t launch_gemv_w4a4(const GemmArgs& a, bool* launched);
+
 // Read and clear the device-side error words of the kernels that wait (gemm.cu, gemm_fused.cu).
 cudaError_t read_and_clear_error_word(unsigned int* out, cudaStream_t stream);
 cudaError_t read_and_clear_error_word_fused(unsigned int* out, cudaStream_t stream);
@@ -96,5 +103,7 @@ cudaError_t read_and_clear_error_word_fused(unsigned int* out, cudaStream_t stre
 // back every copy, for the kernels of gemm.cu and of gemm_fused.cu.  Synchronise the device first.
 cudaError_t set_debug_hooks_gemm(unsigned long long wait_limit_ns, int hold_loads);
 cudaError_t set_debug_hooks_fused(unsigned long long wait_limit_ns, int hold_loads);
+cudaError_t set_debug_hooks_gemv(unsigned long long wait_limit_ns, int hold_loads);
+cudaError_t read_and_clear_error_word_gemv(unsigned int* out, cudaStream_t stream);
 
 }  // namespace qvla
