@@ -736,6 +736,42 @@ qvla_status try_fused(const qvla_layer* L, const void* x, int M, const float* st
   QVLA_CUDA(qvla::launch_gemm_fused(a, launched), "fused linear launch");
   return QVLA_OK;
 }
+
+// Decode-sized batches (M <= 4): one launch of the CUDA-core GEMV that rotates and quantises the
+// activations itself, where the layer allows it (f16/bf16 input and output of one dtype,
+// Hadamard block <= 2048, no per-group step tables, the CTA's working set within its shared
+// memory).  The outputs are those of the rotate-quantise kernel followed by the GEMM, bit for bit.
+qvla_status try_gemv_fused(const qvla_layer* L, const void* x, int M, const float* step_scale, void* y, void* stream,
+                           bool* launched) {
+  *launched = false;
+  if (M > qvla::kGemvMaxM || (step_scale && L->grouped) || L->xdt != L->ydt ||
+      (L->xdt != QVLA_F16 && L->xdt != QVLA_BF16))
+    return QVLA_OK;
+  qvla::GemmArgs a;
+  a.xq = nullptr;
+  a.x_bytes = 3;
+  a.xscale = step_scale;
+  a.xsum = nullptr;
+  a.wq = L->wq;
+  a.wscale = L->wscale;
+  a.wcorr = L->wcorr;
+  a.bias = L->bias;
+  a.y = y;
+  a.ydt = L->ydt;
+  a.acc = nullptr;
+  a.M = M;
+  a.N = L->N;
+  a.K = L->K;
+  a.gated = L->gated;
+  a.x = x;
+  a.xdt = L->xdt;
+  a.log_b = L->log_b;
+  a.inv_sqrt_b = static_cast<float>(1.0 / std::sqrt(static_cast<double>(L->had_block)));
+  a.num_sms = num_sms(L->device);
+  a.stream = static_cast<cudaStream_t>(stream);
+  QVLA_CUDA(qvla::launch_gemv_w4a4(a, launched), "decode linear launch");
+  return QVLA_OK;
+}
 }  // namespace
 
 qvla_status qvla_w4a4_linear_fused(const qvla_layer* L, const void* x, int M, int step, void* y, void* stream) {
@@ -772,6 +808,9 @@ qvla_status qvla_w4a4_linear(const qvla_layer* L, const void* x, int M, int step
   if (qvla_status s = carve_workspace(L, M, workspace, workspace_bytes, &w)) return s;
   const void* xin = nullptr;
   if (qvla_status s = online_input(L, x, M, w, stream, &xin)) return s;
+  bool launched = false;  // one to four tokens: a single launch where the layer allows it
+  if (qvla_status s = try_gemv_fused(L, xin, M, ss, y, stream, &launched)) return s;
+  if (launched) return QVLA_OK;
   if (ss && L->grouped) {  // per-group step scales: per-group codes and sums, promoted per group
     if (qvla_status s = launch_rq(xin, L->xdt, M, L->K, L->had_block, 1, ss, w.xb, w.xscale, nullptr, nullptr, stream, 1,
                                   L->group, w.xgsum))

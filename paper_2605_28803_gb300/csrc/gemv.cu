@@ -55,22 +55,218 @@ struct GvParams {
   int32_t* acc;           // [M][N] or null
   int M, N, K, ldy, nkb, splits;
   float kconst;           // 64 K
+  // kXB 2 (M = 1): the raw activations [1][K] (the output's dtype), rotated and quantised in the
+  // kernel in passes of C channels (a power of two, C | K, b <= C <= 2048); xscale then holds the
+  // step's scale, or is null for a per-token scale, and xsum is unused
+  const void* x;
+  int log_b, C;
+  float inv_sqrt_b;
 };
 
 // The offset-binary bytes q + 8 of a packed word's 8 codes: lo = codes 0, 2, 4, 6, hi = 1, 3, 5, 7
 // (the order in which the rotate-quantise kernel writes its operand bytes).
 __device__ __forceinline__ void unpack8(uint32_t w, uint32_t& lo, uint32_t& hi) { int4x8_to_e4m3_offset(w, lo, hi); }
 
+// kXB 2: the online rotation and the activation quantisation (Sec. 4.1 Eq. 3-5, Sec. 4.2 Eq. 5-6)
+// of this CTA's k-range [kb0, kb1) x 128 of its token, into operand bytes in s_act.  Each pass
+// rotates the C channels containing part of the range with the rotate-quantise kernel's
+// arithmetic stage for stage (butterflies in increasing index-bit order, every sum and difference
+// rounded once), so the rotated values, the scale and the codes are the same bits as that
+// kernel's: thread t loads channels 8 t .. 8 t + 7 of the pass and runs the stages on index bits
+// 0-2 in registers and 3-7 across the lanes; a transpose through shared memory then gives thread
+// t the channels t + 256 w (w < 8), which take the stages on bits 8-10.  The per-token scale takes
+// the largest |value| of the row: where one pass is the whole row (K = C) every CTA has it;
+// otherwise, with K split over a cluster, every CTA sends its range's maximum to every other one.
+// Returns false if that exchange timed out.
+template <int kM, typename XT>
+__device__ __forceinline__ bool rotate_quantize_range(const GvParams& p, const XT* __restrict__ x, int kb0, int kb1,
+                                                      int rank, bool max_exchange, uint8_t* s_act, uint32_t* s_max,
+                                                      uint32_t (*s_maxes)[kM], uint32_t* s_qsum, float2* s_delta,
+                                                      uint32_t bar_max) {
+  const int t = threadIdx.x, lane = t & 31;
+  const int k0 = kb0 * kBK, range = (kb1 - kb0) * kBK;
+  const int rmax = (p.nkb + p.splits - 1) / p.splits * kBK;  // the largest k-range of the cluster
+  float* const s_y = reinterpret_cast<float*>(s_act + static_cast<size_t>(kM) * rmax);  // [kM][range]
+  float* const s_rot = s_y + static_cast<size_t>(kM) * rmax;                            // [C]
+  const int C = p.C, lb = p.log_b;
+  const bool whole_row = p.K == C;
+  for (int m = 0; m < p.M; ++m) {
+    float mx = 0.0f;
+    for (int c = k0 / C; c * C < k0 + range; ++c) {
+      float2 v[4];
+      if (8 * t < C) {
+        rq::Loader<XT>::load(x + static_cast<size_t>(m) * p.K + static_cast<size_t>(c) * C + 8 * t, v);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) v[i] = make_float2(0.0f, 0.0f);
+      }
+      if (lb > 0) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float a = v[i].x, d = v[i].y;
+          v[i] = make_float2(a + d, a - d);
+        }
+      }
+      if (lb > 1) {
+        rq::bfly2(v[0], v[1]);
+        rq::bfly2(v[2], v[3]);
+      }
+      if (lb > 2) {
+        rq::bfly2(v[0], v[2]);
+        rq::bfly2(v[1], v[3]);
+      }
+#pragma unroll
+      for (int bit = 3; bit < 8; ++bit) {
+        if (bit < lb) {  // the lower lane of a pair keeps a + d, the upper one a - d
+          const int mask = 1 << (bit - 3);
+          const float sg = (lane & mask) ? -1.0f : 1.0f;
+          const float2 sg2 = make_float2(sg, sg);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            float2 pv;
+            pv.x = __shfl_xor_sync(0xffffffffu, v[i].x, mask);
+            pv.y = __shfl_xor_sync(0xffffffffu, v[i].y, mask);
+            v[i] = __ffma2_rn(v[i], sg2, pv);
+          }
+        }
+      }
+      __syncthreads();  // the previous pass has read s_rot
+      if (8 * t < C) {
+        reinterpret_cast<float4*>(s_rot)[2 * t] = make_float4(v[0].x, v[0].y, v[1].x, v[1].y);
+        reinterpret_cast<float4*>(s_rot)[2 * t + 1] = make_float4(v[2].x, v[2].y, v[3].x, v[3].y);
+      }
+      __syncthreads();
+      float yv[8];
+#pragma unroll
+      for (int w = 0; w < 8; ++w) yv[w] = t + 256 * w < C ? s_rot[t + 256 * w] : 0.0f;
+#pragma unroll
+      for (int bit = 8; bit < 11; ++bit) {
+        if (bit < lb) {
+          const int h = 1 << (bit - 8);
+#pragma unroll
+          for (int w = 0; w < 8; ++w) {
+            if ((w & h) == 0) {
+              const float a = yv[w], d = yv[w + h];
+              yv[w] = a + d;
+              yv[w + h] = a - d;
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int w = 0; w < 8; ++w) {
+        const int e = t + 256 * w, kk = c * C + e - k0;
+        const bool mine = e < C && kk >= 0 && kk < range;
+        if (mine) s_y[m * range + kk] = yv[w];
+        if (e < C && (mine || whole_row)) mx = fmaxf(mx, fabsf(yv[w]));
+      }
+    }
+    // the warp's largest |value| (non-negative floats order as their bit patterns)
+    const uint32_t wmax = __reduce_max_sync(0xffffffffu, __float_as_uint(mx));
+    if (lane == 0) atomicMax(&s_max[m], wmax);
+  }
+  __syncthreads();  // s_max and s_y are complete
+  bool ok = true;
+  if (max_exchange) {
+    cluster_wait();  // pairs with the arrive at set-up: every CTA's barrier is initialised
+    if (t < p.splits * kM) {
+      const int d = t / kM, mm = t % kM;
+      st_async_u32(mapa_shared(smem_u32(&s_maxes[rank][mm]), static_cast<uint32_t>(d)), s_max[mm],
+                   mapa_shared(bar_max, static_cast<uint32_t>(d)));
+    }
+    ok = mbar_wait_cluster(bar_max, 0);
+  }
+  if (t < kM) {  // the token's scale and the factor of the fast path (0 for a zero scale)
+    float delta;
+    if (p.xscale != nullptr) {
+      delta = __ldg(p.xscale);
+    } else {
+      uint32_t mb = s_max[t];
+      if (max_exchange) {
+        mb = 0u;
+        for (int src = 0; src < p.splits; ++src) mb = max(mb, s_maxes[src][t]);
+      }
+      // max |Z| of the normalised rotation over the row, over q_max = 7
+      delta = __fdiv_rn(__uint_as_float(mb) * p.inv_sqrt_b, 7.0f);
+    }
+    const float rcp = delta > 0.0f ? __fdiv_rn(1.0f, delta) : 0.0f;
+    s_delta[t] = make_float2(delta, p.inv_sqrt_b * rcp);  // cr is infinite exactly when 1 / delta overflows
+  }
+  __syncthreads();
+
+  // codes, every token's groups of 8 at once: the rotate-quantise kernel's fast path, tie band and
+  // exact decision
+  const bool per_step = p.xscale != nullptr;
+  const float2 magic2 = make_float2(rq::kMagic, rq::kMagic), nmagic2 = make_float2(-rq::kMagic, -rq::kMagic);
+  const float2 neg2 = make_float2(-1.0f, -1.0f);
+  const int g8 = range / 8;
+  uint32_t qs[kM];
+#pragma unroll
+  for (int mm = 0; mm < kM; ++mm) qs[mm] = 0u;
+  for (int idx = t; idx < p.M * g8; idx += kGvThreads) {
+    const int m = idx / g8, g = idx - m * g8;
+    const float2 dc = s_delta[m];
+    const float delta = dc.x, cr = dc.y;
+    const float2 cr2 = make_float2(cr, cr);
+    const float4 f0 = reinterpret_cast<const float4*>(s_y + m * range)[2 * g];
+    const float4 f1 = reinterpret_cast<const float4*>(s_y + m * range)[2 * g + 1];
+    const float2 v[4] = {make_float2(f0.x, f0.y), make_float2(f0.z, f0.w), make_float2(f1.x, f1.y),
+                         make_float2(f1.z, f1.w)};
+    float2 u[4];
+    float dev = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float2 tt = __fmul2_rn(v[i], cr2);
+      if (per_step) {
+        tt.x = fminf(fmaxf(tt.x, -7.0f), 7.0f);
+        tt.y = fminf(fmaxf(tt.y, -7.0f), 7.0f);
+      }
+      u[i] = __fadd2_rn(tt, magic2);
+      const float2 d = __ffma2_rn(__fadd2_rn(u[i], nmagic2), neg2, tt);
+      dev = fmaxf(dev, fmaxf(fabsf(d.x), fabsf(d.y)));
+    }
+    if (dev >= rq::kTieBand || isinf(cr)) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        u[i].x = rq::exact_code(v[i].x, p.inv_sqrt_b, delta, cr, 7.0f, rq::kTieBand);
+        u[i].y = rq::exact_code(v[i].y, p.inv_sqrt_b, delta, cr, 7.0f, rq::kTieBand);
+      }
+    }
+    // operand bytes q + 8 in the order k0 k2 k4 k6 k1 k3 k5 k7 of the group
+    const uint32_t lo = (rq::low_bytes(u[0].x, u[1].x, u[2].x, u[3].x) & 0x0F0F0F0Fu) ^ 0x08080808u;
+    const uint32_t hi = (rq::low_bytes(u[0].y, u[1].y, u[2].y, u[3].y) & 0x0F0F0F0Fu) ^ 0x08080808u;
+    reinterpret_cast<uint2*>(s_act + m * range)[g] = make_uint2(lo, hi);
+    const uint32_t q8 = __dp4a(hi, 0x01010101u, __dp4a(lo, 0x01010101u, 0u));
+#pragma unroll
+    for (int mm = 0; mm < kM; ++mm)
+      if (mm == m) qs[mm] += q8;
+  }
+#pragma unroll
+  for (int mm = 0; mm < kM; ++mm) {
+    const uint32_t v = __reduce_add_sync(0xffffffffu, qs[mm]);
+    if (lane == 0 && mm < p.M) atomicAdd(&s_qsum[mm], v);
+  }
+  __syncthreads();  // the operand bytes and code sums are complete
+  return ok;
+}
+
 template <int kM, bool kGated, int kXB, typename OutT>
 __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
   constexpr int kParts = kGated ? 2 : 1;  // 128-row weight groups per CTA
   constexpr int kGvRing = gv_ring<kM, kGated>();
-  constexpr int kActKb = kXB == 1 ? kBK : kBK / 2;  // activation bytes per token and k-block
+  constexpr int kActKb = kXB == 0 ? kBK / 2 : kBK;  // activation bytes per token and k-block
   __shared__ uint32_t s_part[kParts][128][kM];
   // split K: the slices of this CTA's rows from every CTA of the cluster, [source][row][part][m]
   __shared__ uint32_t s_recv[128 * kParts * kM];
   __shared__ __align__(8) uint64_t bar_recv;
-  extern __shared__ __align__(16) uint8_t s_act[];  // [kM][k-range] activation bytes of this CTA
+  // kXB 2: per token, the largest |rotated value| of this CTA's k-range and of every CTA's
+  // (received), the scale, and the sum of the offset codes q + 8 of this CTA's k-range
+  __shared__ uint32_t s_max[kM], s_maxes[8][kM], s_qsum[kM];
+  __shared__ float2 s_delta[kM];  // (scale, 1 / (scale sqrt(b)))
+  __shared__ __align__(8) uint64_t bar_max;
+  // [kM][k-range] activation bytes of this CTA; kXB 2 then [kM][k-range] float rotated values
+  // and one pass of C floats
+  extern __shared__ __align__(16) uint8_t s_act[];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int S = p.splits;
@@ -82,13 +278,19 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
   const int R = 128 / S;  // rows this CTA finishes: [rank R, (rank + 1) R)
 
   for (int i = threadIdx.x; i < kParts * 128 * kM; i += kGvThreads) (&s_part[0][0][0])[i] = 0u;
+  if (kXB == 2 && threadIdx.x < kM) s_max[threadIdx.x] = s_qsum[threadIdx.x] = 0u;
+  // kXB 2 with per-token scales: the CTAs of the cluster exchange their k-ranges' maxima
+  // (unless one rotation pass is the whole row, which every CTA then rotates)
+  const bool max_exchange = kXB == 2 && S > 1 && p.xscale == nullptr && p.K > p.C;
   if (S > 1) {
     // every CTA of the cluster sends this one its partials of these rows; the cluster barrier
     // completed before the first send guarantees every receiver's barrier exists
     if (threadIdx.x == 0) {
       mbar_init(smem_u32(&bar_recv), 1);
+      if (max_exchange) mbar_init(smem_u32(&bar_max), 1);
       mbar_init_fence();
       mbar_arrive_expect_tx(smem_u32(&bar_recv), static_cast<uint32_t>(S * R * kParts * kM * 4));
+      if (max_exchange) mbar_arrive_expect_tx(smem_u32(&bar_max), static_cast<uint32_t>(S * kM * 4));
     }
     cluster_arrive_relaxed();
   }
@@ -110,17 +312,13 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
     const int kb = kb0 + kpar + kGvPhases * i;
     if (kb < kb1) load_w(kb, ring[i]);  // the weights no earlier kernel writes: before the wait
   }
-  griddep_wait();  // the activations, their scales and sums come from the previous kernel
-  if (threadIdx.x == 0) griddep_launch_dependents();
-  // the epilogue's parameters of this thread's (row, token) entries, fetched while the weights stream
+  // the epilogue's parameters of this thread's (row, token) entries: the layer's, before the wait
   constexpr int kEnt = (128 * kM + kGvThreads - 1) / kGvThreads;
   float e_cm[kEnt], e_xs[kEnt], e_wc[kEnt][kParts], e_ws[kEnt][kParts], e_bs[kEnt][kParts];
 #pragma unroll
   for (int u = 0; u < kEnt; ++u) {
     const int e = threadIdx.x + u * kGvThreads;
-    const int row = rank * R + min(e, R * kM - 1) / kM, m = min(e % kM, p.M - 1);
-    e_cm[u] = 8.0f * static_cast<float>(p.xsum[m]) + p.kconst;
-    e_xs[u] = p.xscale[m];
+    const int row = rank * R + min(e, R * kM - 1) / kM;
 #pragma unroll
     for (int part = 0; part < kParts; ++part) {
       const int n = kGated ? 2 * unit * 128 + part * 128 + row : min(unit * 128 + row, p.N - 1);
@@ -129,15 +327,35 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
       e_bs[u][part] = __ldg(p.bias + n);
     }
   }
-  {  // this CTA's k-range of every token's activation bytes, once, into shared memory
+  griddep_wait();  // the activations, their scales and sums come from the previous kernel
+  if (threadIdx.x == 0) griddep_launch_dependents();
+#pragma unroll
+  for (int u = 0; u < kEnt; ++u) {
+    const int m = min((threadIdx.x + u * kGvThreads) % kM, p.M - 1);
+    if constexpr (kXB == 2) {  // the activations' code sums are taken out of the partial sums
+      e_cm[u] = p.kconst;
+      e_xs[u] = 0.0f;
+    } else {
+      e_cm[u] = 8.0f * static_cast<float>(p.xsum[m]) + p.kconst;
+      e_xs[u] = p.xscale[m];
+    }
+  }
+  bool landed = true, cluster_waited = false;
+  if constexpr (kXB == 2) {
+    landed = rotate_quantize_range<kM>(p, static_cast<const OutT*>(p.x), kb0, kb1, rank, max_exchange, s_act, s_max,
+                                       s_maxes, s_qsum, s_delta, smem_u32(&bar_max));
+    cluster_waited = max_exchange;
+#pragma unroll
+    for (int u = 0; u < kEnt; ++u) e_xs[u] = s_delta[min((threadIdx.x + u * kGvThreads) % kM, p.M - 1)].x;
+  } else {  // this CTA's k-range of every token's activation bytes, once, into shared memory
     const int row16 = (kb1 - kb0) * kActKb / 16;  // 16-byte pieces per token
     for (int i = threadIdx.x; i < p.M * row16; i += kGvThreads) {
       const int m = i / row16, c = i % row16;
       reinterpret_cast<uint4*>(s_act)[m * row16 + c] = __ldg(reinterpret_cast<const uint4*>(
           p.xq + static_cast<size_t>(m) * (p.K / (kBK / kActKb)) + kb0 * kActKb) + c);
     }
+    __syncthreads();
   }
-  __syncthreads();
 
   uint32_t acc[kParts][4][kM];
 #pragma unroll
@@ -158,7 +376,7 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
         for (int m = 0; m < kM; ++m) {
           if (m < p.M) {
             const uint8_t* arow = s_act + (static_cast<size_t>(m) * (kb1 - kb0) + (kb - kb0)) * kActKb;
-            if constexpr (kXB == 1) {
+            if constexpr (kXB != 0) {
               const uint4* src = reinterpret_cast<const uint4*>(arow + q * 32);
               const uint4 v0 = src[0], v1 = src[1];
               alo[m][0] = v0.x; ahi[m][0] = v0.y; alo[m][1] = v0.z; ahi[m][1] = v0.w;
@@ -217,19 +435,24 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
         for (int m = 0; m < kM; ++m) atomicAdd(&s_part[part][slice * 32 + 8 * t + lane / 4][m], acc[part][t][m]);
   }
   __syncthreads();
-  bool landed = true;
+  // kXB 2: 8 x the activation codes' sum over this CTA's k-range, taken out of its partials
+  // (the sums of all ranks then hold S - 8 sum_k q_x, a signed value in 32-bit wrap-around)
+  auto xcorr = [&](int m) -> uint32_t {
+    if constexpr (kXB == 2) return 8u * s_qsum[m] - 64u * static_cast<uint32_t>((kb1 - kb0) * kBK);
+    return 0u;
+  };
   if (S > 1) {
-    cluster_wait();  // pairs with the arrive at set-up: every receive barrier is initialised
+    if (!cluster_waited) cluster_wait();  // pairs with the arrive at set-up: every receive barrier is initialised
     // each partial goes to the CTA that finishes its row, as an asynchronous store completing on
     // that CTA's barrier; no CTA reads another's shared memory, so none waits for the others to leave
     for (int i = threadIdx.x; i < 128 * kParts * kM; i += kGvThreads) {
       const int row = i / (kParts * kM), part = (i / kM) % kParts, m = i % kM;
       const int d = row / R;
       const uint32_t dst = smem_u32(&s_recv[((rank * R + (row - d * R)) * kParts + part) * kM + m]);
-      st_async_u32(mapa_shared(dst, static_cast<uint32_t>(d)), s_part[part][row][m],
+      st_async_u32(mapa_shared(dst, static_cast<uint32_t>(d)), s_part[part][row][m] - xcorr(m),
                    mapa_shared(smem_u32(&bar_recv), static_cast<uint32_t>(d)));
     }
-    landed = mbar_wait_cluster(smem_u32(&bar_recv), 0);
+    landed = mbar_wait_cluster(smem_u32(&bar_recv), 0) && landed;
   }
 
   // rank r finishes rows [r R, (r + 1) R) of the group(s), adding every rank's partial
@@ -246,14 +469,14 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
         sum[part] = 0u;
         for (int src = 0; src < S; ++src) sum[part] += s_recv[((src * R + rr) * kParts + part) * kM + m];
       } else {
-        sum[part] = s_part[part][row][m];
+        sum[part] = s_part[part][row][m] - xcorr(m);
       }
     }
     // the epilogue of the tensor-core path: exact accumulator, one float32 scale product, fma, one rounding
     if constexpr (!kGated) {
       const int n = unit * 128 + row;
       if (n < p.N) {
-        const float a = static_cast<float>(sum[0]) - (e_cm[u] + e_wc[u][0]);
+        const float a = static_cast<float>(static_cast<int32_t>(sum[0])) - (e_cm[u] + e_wc[u][0]);
         reinterpret_cast<OutT*>(p.y)[static_cast<size_t>(m) * p.ldy + n] = to_out<OutT>(fmaf(a, e_xs[u] * e_ws[u][0], e_bs[u][0]));
         if (p.acc) p.acc[static_cast<size_t>(m) * p.N + n] = static_cast<int32_t>(a);
       }
@@ -261,8 +484,8 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
       // weight rows 256 unit + row (gate) and + 128 (up) of hidden unit j; h = gelu(gate) * up
       const int H = p.N / 2, j = unit * 128 + row;
       if (j < H) {
-        const float ag = static_cast<float>(sum[0]) - (e_cm[u] + e_wc[u][0]);
-        const float au = static_cast<float>(sum[1]) - (e_cm[u] + e_wc[u][1]);
+        const float ag = static_cast<float>(static_cast<int32_t>(sum[0])) - (e_cm[u] + e_wc[u][0]);
+        const float au = static_cast<float>(static_cast<int32_t>(sum[1])) - (e_cm[u] + e_wc[u][1]);
         const float2 gu = unpack2<OutT>(pack2<OutT>(fmaf(ag, e_xs[u] * e_ws[u][0], e_bs[u][0]),
                                                     fmaf(au, e_xs[u] * e_ws[u][1], e_bs[u][1])));
         reinterpret_cast<OutT*>(p.y)[static_cast<size_t>(m) * p.ldy + j] = to_out<OutT>(gelu_tanh(gu.x) * gu.y);
@@ -278,10 +501,11 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
 template <int kM, bool kGated, int kXB, typename OutT>
 cudaError_t launch_gv(const GemmArgs& a, GvParams p, int units) {
   auto kern = gemv_w4a4_kernel<kM, kGated, kXB, OutT>;
-  // the largest k-range of a CTA, for every token
-  const size_t act = static_cast<size_t>(kM) * ((p.nkb + p.splits - 1) / p.splits) * (kXB == 1 ? kBK : kBK / 2);
+  // the largest k-range of a CTA, for every token (kXB 2: and its rotated values, and one pass)
+  size_t act = static_cast<size_t>(kM) * ((p.nkb + p.splits - 1) / p.splits) * (kXB == 0 ? kBK / 2 : kBK);
+  if (kXB == 2) act = 5 * act + 4 * static_cast<size_t>(p.C);
   if (act > static_cast<size_t>(kGemvActMax)) return kNotApplicable;
-  if (act > 48 * 1024) {
+  if (act + 16 * 1024 > 48 * 1024) {  // with the static shared memory (up to 8.4 KB) past the default 48 KB
     cudaError_t e = prepare_kernel(reinterpret_cast<const void*>(kern), kGemvActMax);
     if (e != cudaSuccess) return e == kNotApplicable ? cudaErrorUnknown : e;
   }
@@ -307,8 +531,12 @@ cudaError_t launch_gv(const GemmArgs& a, GvParams p, int units) {
 template <bool kGated, int kXB, typename OutT>
 cudaError_t launch_gv_m(const GemmArgs& a, const GvParams& p, int units) {
   if (a.M == 1) return launch_gv<1, kGated, kXB, OutT>(a, p, units);
-  if (a.M == 2) return launch_gv<2, kGated, kXB, OutT>(a, p, units);
-  return launch_gv<4, kGated, kXB, OutT>(a, p, units);
+  if constexpr (kXB == 2) {
+    return kNotApplicable;  // the one-launch linear takes one token
+  } else {
+    if (a.M == 2) return launch_gv<2, kGated, kXB, OutT>(a, p, units);
+    return launch_gv<4, kGated, kXB, OutT>(a, p, units);
+  }
 }
 
 template <int kXB, typename OutT>
@@ -333,7 +561,12 @@ cudaError_t set_debug_hooks_gemv(unsigned long long wait_limit_ns, int hold_load
 
 cudaError_t launch_gemv_w4a4(const GemmArgs& a, bool* launched) {
   *launched = false;
-  if (a.M < 1 || a.M > kGemvMaxM || a.gscale || (a.x_bytes != 0 && a.x_bytes != 1)) return cudaSuccess;
+  if (a.M < 1 || a.M > kGemvMaxM || a.gscale || (a.x_bytes != 0 && a.x_bytes != 1 && a.x_bytes != 3)) return cudaSuccess;
+  // raw activations (one token): rotation passes of C channels, C the largest power of two up to
+  // 2048 that divides K, holding whole Hadamard blocks; x of the output's dtype
+  int C = 2048;
+  while (a.K % C != 0) C /= 2;
+  if (a.x_bytes == 3 && (a.M != 1 || a.xdt != a.ydt || a.log_b < 0 || (1 << a.log_b) > C)) return cudaSuccess;
   GvParams p;
   p.wq = a.wq;
   p.xq = a.xq;
@@ -350,14 +583,27 @@ cudaError_t launch_gemv_w4a4(const GemmArgs& a, bool* launched) {
   p.ldy = a.gated ? a.N / 2 : a.N;
   p.nkb = a.K / kBK;
   p.kconst = 64.0f * static_cast<float>(a.K);
+  p.x = a.x;
+  p.log_b = a.log_b;
+  p.C = C;
+  p.inv_sqrt_b = a.inv_sqrt_b;
   // one CTA per 128-row group (gated: per 128 hidden units, gate and up), K split over a cluster
   // of up to 8 until the grid holds about two CTAs per SM
   const int units = a.gated ? a.N / 256 : (a.N + 127) / 128;
   int splits = 1;
   while (splits < 8 && 2 * splits <= p.nkb && units * splits < 2 * a.num_sms) splits *= 2;
   p.splits = splits;
-  cudaError_t e = a.x_bytes == 1 ? (a.ydt == 0 ? launch_gv_g<1, __half>(a, p, units) : launch_gv_g<1, __nv_bfloat16>(a, p, units))
-                                 : (a.ydt == 0 ? launch_gv_g<0, __half>(a, p, units) : launch_gv_g<0, __nv_bfloat16>(a, p, units));
+  // raw activations: the CTAs' rotations and quantisation sit between the previous kernel and
+  // the weights' use, once per CTA; with more than about 1.25 CTAs per SM the rotate-quantise
+  // kernel ahead of the GEMV (its work overlapping the GEMV's weight loads) is measured faster
+  if (a.x_bytes == 3 && 4 * units * splits > 5 * a.num_sms) return cudaSuccess;
+  cudaError_t e;
+  if (a.x_bytes == 3)
+    e = a.ydt == 0 ? launch_gv_g<2, __half>(a, p, units) : launch_gv_g<2, __nv_bfloat16>(a, p, units);
+  else if (a.x_bytes == 1)
+    e = a.ydt == 0 ? launch_gv_g<1, __half>(a, p, units) : launch_gv_g<1, __nv_bfloat16>(a, p, units);
+  else
+    e = a.ydt == 0 ? launch_gv_g<0, __half>(a, p, units) : launch_gv_g<0, __nv_bfloat16>(a, p, units);
   if (e == kNotApplicable) return cudaSuccess;  // the activations of a CTA would not fit
   *launched = e == cudaSuccess;
   return e;
