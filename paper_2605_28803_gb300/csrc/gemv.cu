@@ -593,10 +593,14 @@ cudaError_t launch_gemv_w4a4(const GemmArgs& a, bool* launched) {
   int splits = 1;
   while (splits < 8 && 2 * splits <= p.nkb && units * splits < 2 * a.num_sms) splits *= 2;
   p.splits = splits;
-  // raw activations: the CTAs' rotations and quantisation sit between the previous kernel and
-  // the weights' use, once per CTA; with more than about 1.25 CTAs per SM the rotate-quantise
-  // kernel ahead of the GEMV (its work overlapping the GEMV's weight loads) is measured faster
-  if (a.x_bytes == 3 && 4 * units * splits > 5 * a.num_sms) return cudaSuccess;
+  // raw activations: the CTAs' rotation and quantisation sit between the previous kernel and the
+  // weights' use.  Where the grid holds more than about 1.25 CTAs per SM and a CTA's weights do
+  // not all fit in the loads it issues before the wait, the rotate-quantise kernel ahead of the
+  // GEMV (its work overlapping the GEMV's first weight loads) measured faster.
+  if (a.x_bytes == 3) {
+    const int ring = (a.gated ? gv_ring<1, true>() : gv_ring<1, false>()) * kGvPhases;
+    if (4 * units * splits > 5 * a.num_sms && (p.nkb + splits - 1) / splits >= ring) return cudaSuccess;
+  }
   cudaError_t e;
   if (a.x_bytes == 3)
     e = a.ydt == 0 ? launch_gv_g<2, __half>(a, p, units) : launch_gv_g<2, __nv_bfloat16>(a, p, units);

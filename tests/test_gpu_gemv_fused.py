@@ -64,7 +64,7 @@ def _input(rng, M, K, dt):
 
 
 SHAPES = [(2048, 2560, 2048), (16384, 2048, 2048), (1024, 1024, 64), (384, 272, 128), (3072, 512, 1024), (2048, 128, 1),
-          (16384, 16, 512)]
+          (16384, 16, 512), (1024, 4096, 1024)]
 
 
 @pytest.mark.parametrize("dt", ["f16", "bf16"])
@@ -99,7 +99,8 @@ def test_one_launch_equals_two_launch_per_step(dt, K, N, had):
 @pytest.mark.parametrize("K,N,had,M", [(4096, 256, 4096, 1), (2048, 2560, 2048, 2), (2048, 20480, 2048, 1)])
 def test_layers_outside_the_one_launch_take_two(K, N, had, M):
     """A Hadamard block wider than one pass, more than one token, or a grid of more than about
-    1.25 CTAs per SM: the two launches run (the workspace is written), with the same result."""
+    1.25 CTAs per SM whose CTAs cannot load all their weights ahead of the previous kernel's end:
+    the two launches run (the workspace is written), with the same result."""
     rng = np.random.default_rng(K + N + M)
     layer, _, _, _ = _layer(rng, N, K, had, "bf16", bias=False)
     x = _input(rng, M, K, "bf16")
