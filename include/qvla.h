@@ -262,10 +262,10 @@ size_t qvla_linear_workspace_bytes(const qvla_layer* layer, int M);
  * qvla_linear_workspace_bytes(layer, M) bytes, 256-byte aligned, used only during the call's
  * kernels on `stream` (calls that overlap on the GPU must not share it).
  * One token (M = 1, the decode step) runs as a single kernel where the layer allows it (f16 or
- * bf16 input of the output's dtype, Hadamard block <= 2048, no per-group step table, about one
- * CTA per SM): a GEMV whose CTAs rotate and quantise their share of x themselves, with the same
- * results bit for bit; the workspace is then not touched unless the layer has an online
- * rotation. */
+ * bf16 input of the output's dtype, Hadamard block <= 2048, no per-group step table, a split of
+ * K whose CTAs each see at most two 2048-channel rotation passes): a GEMV whose CTAs rotate and
+ * quantise their share of x themselves, with the same results bit for bit; the workspace is
+ * then not touched unless the layer has an online rotation. */
 qvla_status qvla_w4a4_linear(const qvla_layer* layer, const void* x, int M, int step, void* y,
                              void* workspace, size_t workspace_bytes, void* stream);
 

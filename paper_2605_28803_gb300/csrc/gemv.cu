@@ -29,10 +29,12 @@ constexpr int kGemvActMax = 96 * 1024;  // shared memory for a CTA's activation 
 constexpr int kGvPhases = kGvThreads / 32 / 4;
 
 // k-blocks of weight loads a warp keeps in flight: 64 KB per CTA at one token, 32 KB where the
-// accumulators of more tokens (or of a gated layer's two groups) need the registers
-template <int kM, bool kGated>
+// accumulators of more tokens (or of a gated layer's two groups) need the registers.  The
+// one-launch linear (kXB 2, one token) runs about one CTA per SM or fewer, whose registers allow
+// a gated layer 96 KB.
+template <int kM, bool kGated, int kXB>
 __host__ __device__ constexpr int gv_ring() {
-  return kM == 1 ? (kGated ? 2 : 4) : 2;
+  return kM == 1 ? (kGated ? (kXB == 2 ? 6 : 2) : 4) : 2;
 }
 
 // Four bytes into the shared memory of a CTA of the cluster, completing 4 bytes of the
@@ -68,201 +70,171 @@ struct GvParams {
 __device__ __forceinline__ void unpack8(uint32_t w, uint32_t& lo, uint32_t& hi) { int4x8_to_e4m3_offset(w, lo, hi); }
 
 // kXB 2: the online rotation and the activation quantisation (Sec. 4.1 Eq. 3-5, Sec. 4.2 Eq. 5-6)
-// of this CTA's k-range [kb0, kb1) x 128 of its token, into operand bytes in s_act.  Each pass
-// rotates the C channels containing part of the range with the rotate-quantise kernel's
-// arithmetic stage for stage (butterflies in increasing index-bit order, every sum and difference
-// rounded once), so the rotated values, the scale and the codes are the same bits as that
-// kernel's: thread t loads channels 8 t .. 8 t + 7 of the pass and runs the stages on index bits
-// 0-2 in registers and 3-7 across the lanes; a transpose through shared memory then gives thread
-// t the channels t + 256 w (w < 8), which take the stages on bits 8-10.  The per-token scale takes
-// the largest |value| of the row: where one pass is the whole row (K = C) every CTA has it;
+// of one token's k-range [kb0, kb1) x 128 in this CTA, into operand bytes in s_act.  Each of the
+// (at most kGvPasses) passes rotates the C channels containing part of the range with the
+// rotate-quantise kernel's arithmetic stage for stage (butterflies in increasing index-bit order,
+// every sum and difference rounded once), so the rotated values, the scale and the codes are the
+// same bits as that kernel's: thread t loads channels 8 t .. 8 t + 7 of the pass and runs the
+// stages on index bits 0-2 in registers and 3-7 across the lanes; a transpose through shared
+// memory then gives thread t the channels t + 256 w (w < 8), which take the stages on bits 8-10
+// and stay in its registers.  The per-token scale
+// takes the largest |value| of the row: where one pass is the whole row (K = C) every CTA has it;
 // otherwise, with K split over a cluster, every CTA sends its range's maximum to every other one.
-// Returns false if that exchange timed out.
-template <int kM, typename XT>
-__device__ __forceinline__ bool rotate_quantize_range(const GvParams& p, const XT* __restrict__ x, int kb0, int kb1,
-                                                      int rank, bool max_exchange, uint8_t* s_act, uint32_t* s_max,
-                                                      uint32_t (*s_maxes)[kM], uint32_t* s_qsum, float2* s_delta,
-                                                      uint32_t bar_max) {
-  const int t = threadIdx.x, lane = t & 31;
+// Each thread then turns its values of the range into codes (the rotate-quantise kernel's fast
+// path, tie band and exact decision, value by value) and stores their operand bytes.  Returns
+// the scale in *delta_out, the sum of the range's offset codes q + 8 in s_wsum (one partial per
+// warp), and false if a wait timed out.
+constexpr int kGvPasses = 2;
+template <typename XT>
+__device__ __forceinline__ bool rotate_quantize_token(const GvParams& p, const XT* __restrict__ x, int kb0, int kb1,
+                                                      int rank, bool max_exchange, uint8_t* s_act, uint32_t* s_wmax,
+                                                      uint32_t* s_maxes, uint32_t* s_wsum, uint32_t bar_max,
+                                                      float* delta_out) {
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const int k0 = kb0 * kBK, range = (kb1 - kb0) * kBK;
   const int rmax = (p.nkb + p.splits - 1) / p.splits * kBK;  // the largest k-range of the cluster
-  float* const s_y = reinterpret_cast<float*>(s_act + static_cast<size_t>(kM) * rmax);  // [kM][range]
-  float* const s_rot = s_y + static_cast<size_t>(kM) * rmax;                            // [C]
   const int C = p.C, lb = p.log_b;
+  float* const s_rot = reinterpret_cast<float*>(s_act + rmax);  // [C]
   const bool whole_row = p.K == C;
-  for (int m = 0; m < p.M; ++m) {
-    float mx = 0.0f;
-    for (int c = k0 / C; c * C < k0 + range; ++c) {
-      float2 v[4];
-      if (8 * t < C) {
-        rq::Loader<XT>::load(x + static_cast<size_t>(m) * p.K + static_cast<size_t>(c) * C + 8 * t, v);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) v[i] = make_float2(0.0f, 0.0f);
-      }
-      if (lb > 0) {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float a = v[i].x, d = v[i].y;
-          v[i] = make_float2(a + d, a - d);
-        }
-      }
-      if (lb > 1) {
-        rq::bfly2(v[0], v[1]);
-        rq::bfly2(v[2], v[3]);
-      }
-      if (lb > 2) {
-        rq::bfly2(v[0], v[2]);
-        rq::bfly2(v[1], v[3]);
-      }
-#pragma unroll
-      for (int bit = 3; bit < 8; ++bit) {
-        if (bit < lb) {  // the lower lane of a pair keeps a + d, the upper one a - d
-          const int mask = 1 << (bit - 3);
-          const float sg = (lane & mask) ? -1.0f : 1.0f;
-          const float2 sg2 = make_float2(sg, sg);
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            float2 pv;
-            pv.x = __shfl_xor_sync(0xffffffffu, v[i].x, mask);
-            pv.y = __shfl_xor_sync(0xffffffffu, v[i].y, mask);
-            v[i] = __ffma2_rn(v[i], sg2, pv);
-          }
-        }
-      }
-      __syncthreads();  // the previous pass has read s_rot
-      if (8 * t < C) {
-        reinterpret_cast<float4*>(s_rot)[2 * t] = make_float4(v[0].x, v[0].y, v[1].x, v[1].y);
-        reinterpret_cast<float4*>(s_rot)[2 * t + 1] = make_float4(v[2].x, v[2].y, v[3].x, v[3].y);
-      }
-      __syncthreads();
-      float yv[8];
-#pragma unroll
-      for (int w = 0; w < 8; ++w) yv[w] = t + 256 * w < C ? s_rot[t + 256 * w] : 0.0f;
-#pragma unroll
-      for (int bit = 8; bit < 11; ++bit) {
-        if (bit < lb) {
-          const int h = 1 << (bit - 8);
-#pragma unroll
-          for (int w = 0; w < 8; ++w) {
-            if ((w & h) == 0) {
-              const float a = yv[w], d = yv[w + h];
-              yv[w] = a + d;
-              yv[w + h] = a - d;
-            }
-          }
-        }
-      }
-#pragma unroll
-      for (int w = 0; w < 8; ++w) {
-        const int e = t + 256 * w, kk = c * C + e - k0;
-        const bool mine = e < C && kk >= 0 && kk < range;
-        if (mine) s_y[m * range + kk] = yv[w];
-        if (e < C && (mine || whole_row)) mx = fmaxf(mx, fabsf(yv[w]));
-      }
-    }
-    // the warp's largest |value| (non-negative floats order as their bit patterns)
-    const uint32_t wmax = __reduce_max_sync(0xffffffffu, __float_as_uint(mx));
-    if (lane == 0) atomicMax(&s_max[m], wmax);
-  }
-  __syncthreads();  // s_max and s_y are complete
+  const int c0 = k0 / C, passes = (k0 + range + C - 1) / C - c0;
   bool ok = true;
-  if (max_exchange) {
-    cluster_wait();  // pairs with the arrive at set-up: every CTA's barrier is initialised
-    if (t < p.splits * kM) {
-      const int d = t / kM, mm = t % kM;
-      st_async_u32(mapa_shared(smem_u32(&s_maxes[rank][mm]), static_cast<uint32_t>(d)), s_max[mm],
-                   mapa_shared(bar_max, static_cast<uint32_t>(d)));
-    }
-    ok = mbar_wait_cluster(bar_max, 0);
-  }
-  if (t < kM) {  // the token's scale and the factor of the fast path (0 for a zero scale)
-    float delta;
-    if (p.xscale != nullptr) {
-      delta = __ldg(p.xscale);
+  float yv[kGvPasses][8];
+  float mx = 0.0f;
+#pragma unroll
+  for (int ps = 0; ps < kGvPasses; ++ps) {
+    if (ps >= passes) break;
+    const int c = c0 + ps;
+    float2 v[4];
+    if (8 * t < C) {
+      rq::Loader<XT>::load(x + static_cast<size_t>(c) * C + 8 * t, v);
     } else {
-      uint32_t mb = s_max[t];
-      if (max_exchange) {
-        mb = 0u;
-        for (int src = 0; src < p.splits; ++src) mb = max(mb, s_maxes[src][t]);
-      }
-      // max |Z| of the normalised rotation over the row, over q_max = 7
-      delta = __fdiv_rn(__uint_as_float(mb) * p.inv_sqrt_b, 7.0f);
-    }
-    const float rcp = delta > 0.0f ? __fdiv_rn(1.0f, delta) : 0.0f;
-    s_delta[t] = make_float2(delta, p.inv_sqrt_b * rcp);  // cr is infinite exactly when 1 / delta overflows
-  }
-  __syncthreads();
-
-  // codes, every token's groups of 8 at once: the rotate-quantise kernel's fast path, tie band and
-  // exact decision
-  const bool per_step = p.xscale != nullptr;
-  const float2 magic2 = make_float2(rq::kMagic, rq::kMagic), nmagic2 = make_float2(-rq::kMagic, -rq::kMagic);
-  const float2 neg2 = make_float2(-1.0f, -1.0f);
-  const int g8 = range / 8;
-  uint32_t qs[kM];
 #pragma unroll
-  for (int mm = 0; mm < kM; ++mm) qs[mm] = 0u;
-  for (int idx = t; idx < p.M * g8; idx += kGvThreads) {
-    const int m = idx / g8, g = idx - m * g8;
-    const float2 dc = s_delta[m];
-    const float delta = dc.x, cr = dc.y;
-    const float2 cr2 = make_float2(cr, cr);
-    const float4 f0 = reinterpret_cast<const float4*>(s_y + m * range)[2 * g];
-    const float4 f1 = reinterpret_cast<const float4*>(s_y + m * range)[2 * g + 1];
-    const float2 v[4] = {make_float2(f0.x, f0.y), make_float2(f0.z, f0.w), make_float2(f1.x, f1.y),
-                         make_float2(f1.z, f1.w)};
-    float2 u[4];
-    float dev = 0.0f;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float2 tt = __fmul2_rn(v[i], cr2);
-      if (per_step) {
-        tt.x = fminf(fmaxf(tt.x, -7.0f), 7.0f);
-        tt.y = fminf(fmaxf(tt.y, -7.0f), 7.0f);
-      }
-      u[i] = __fadd2_rn(tt, magic2);
-      const float2 d = __ffma2_rn(__fadd2_rn(u[i], nmagic2), neg2, tt);
-      dev = fmaxf(dev, fmaxf(fabsf(d.x), fabsf(d.y)));
+      for (int i = 0; i < 4; ++i) v[i] = make_float2(0.0f, 0.0f);
     }
-    if (dev >= rq::kTieBand || isinf(cr)) {
+    if (lb > 0) {
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        u[i].x = rq::exact_code(v[i].x, p.inv_sqrt_b, delta, cr, 7.0f, rq::kTieBand);
-        u[i].y = rq::exact_code(v[i].y, p.inv_sqrt_b, delta, cr, 7.0f, rq::kTieBand);
+        const float a = v[i].x, d = v[i].y;
+        v[i] = make_float2(a + d, a - d);
       }
     }
-    // operand bytes q + 8 in the order k0 k2 k4 k6 k1 k3 k5 k7 of the group
-    const uint32_t lo = (rq::low_bytes(u[0].x, u[1].x, u[2].x, u[3].x) & 0x0F0F0F0Fu) ^ 0x08080808u;
-    const uint32_t hi = (rq::low_bytes(u[0].y, u[1].y, u[2].y, u[3].y) & 0x0F0F0F0Fu) ^ 0x08080808u;
-    reinterpret_cast<uint2*>(s_act + m * range)[g] = make_uint2(lo, hi);
-    const uint32_t q8 = __dp4a(hi, 0x01010101u, __dp4a(lo, 0x01010101u, 0u));
+    if (lb > 1) {
+      rq::bfly2(v[0], v[1]);
+      rq::bfly2(v[2], v[3]);
+    }
+    if (lb > 2) {
+      rq::bfly2(v[0], v[2]);
+      rq::bfly2(v[1], v[3]);
+    }
 #pragma unroll
-    for (int mm = 0; mm < kM; ++mm)
-      if (mm == m) qs[mm] += q8;
-  }
+    for (int bit = 3; bit < 8; ++bit) {
+      if (bit < lb) {  // the lower lane of a pair keeps a + d, the upper one a - d
+        const int mask = 1 << (bit - 3);
+        const float sg = (lane & mask) ? -1.0f : 1.0f;
+        const float2 sg2 = make_float2(sg, sg);
 #pragma unroll
-  for (int mm = 0; mm < kM; ++mm) {
-    const uint32_t v = __reduce_add_sync(0xffffffffu, qs[mm]);
-    if (lane == 0 && mm < p.M) atomicAdd(&s_qsum[mm], v);
+        for (int i = 0; i < 4; ++i) {
+          float2 pv;
+          pv.x = __shfl_xor_sync(0xffffffffu, v[i].x, mask);
+          pv.y = __shfl_xor_sync(0xffffffffu, v[i].y, mask);
+          v[i] = __ffma2_rn(v[i], sg2, pv);
+        }
+      }
+    }
+    if (ps > 0) __syncthreads();  // the previous pass has read s_rot
+    if (8 * t < C) {
+      reinterpret_cast<float4*>(s_rot)[2 * t] = make_float4(v[0].x, v[0].y, v[1].x, v[1].y);
+      reinterpret_cast<float4*>(s_rot)[2 * t + 1] = make_float4(v[2].x, v[2].y, v[3].x, v[3].y);
+    }
+    __syncthreads();
+    float* const yp = yv[ps];
+#pragma unroll
+    for (int w = 0; w < 8; ++w) yp[w] = t + 256 * w < C ? s_rot[t + 256 * w] : 0.0f;
+#pragma unroll
+    for (int bit = 8; bit < 11; ++bit) {
+      if (bit < lb) {
+        const int h = 1 << (bit - 8);
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+          if ((w & h) == 0) {
+            const float a = yp[w], d = yp[w + h];
+            yp[w] = a + d;
+            yp[w + h] = a - d;
+          }
+        }
+      }
+    }
+    float m8[8];  // |values| that count towards the maximum, reduced as a tree
+#pragma unroll
+    for (int w = 0; w < 8; ++w) {
+      const int e = t + 256 * w, kk = c * C + e - k0;
+      m8[w] = (e < C && (whole_row || (kk >= 0 && kk < range))) ? fabsf(yp[w]) : 0.0f;
+    }
+    mx = fmaxf(mx, fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])), fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7]))));
   }
+  // the CTA's largest |value| (non-negative floats order as their bit patterns): one per warp
+  const uint32_t wmax = __reduce_max_sync(0xffffffffu, __float_as_uint(mx));
+  if (lane == 0) s_wmax[warp] = wmax;
+  __syncthreads();
+  uint32_t cmax = 0u;
+#pragma unroll
+  for (int i = 0; i < kGvThreads / 32; ++i) cmax = max(cmax, s_wmax[i]);
+  if (max_exchange) {
+    cluster_wait();  // pairs with the arrive at set-up: every CTA's barrier is initialised
+    if (t < p.splits)
+      st_async_u32(mapa_shared(smem_u32(&s_maxes[rank]), static_cast<uint32_t>(t)), cmax,
+                   mapa_shared(bar_max, static_cast<uint32_t>(t)));
+    ok = mbar_wait_cluster(bar_max, 0) && ok;
+    cmax = 0u;
+    for (int src = 0; src < p.splits; ++src) cmax = max(cmax, s_maxes[src]);
+  }
+  const bool per_step = p.xscale != nullptr;
+  // the scale: the step's, or max |Z| of the normalised rotation over the row over q_max = 7
+  const float delta = per_step ? __ldg(p.xscale) : __fdiv_rn(__uint_as_float(cmax) * p.inv_sqrt_b, 7.0f);
+  const float cr = p.inv_sqrt_b * (delta > 0.0f ? __fdiv_rn(1.0f, delta) : 0.0f);  // infinite iff 1 / delta overflows
+  *delta_out = delta;
+  // codes of this thread's channels of the range: operand byte q + 8 of channel k at byte
+  // 8 (k / 8) + j of the range, j = i / 2 for the even i = k % 8 and 4 + i / 2 for the odd
+  uint32_t qs = 0u;
+#pragma unroll
+  for (int ps = 0; ps < kGvPasses; ++ps) {
+    if (ps >= passes) break;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) {
+      const int e = t + 256 * w, kk = (c0 + ps) * C + e - k0;
+      if (e < C && kk >= 0 && kk < range) {
+        const float y = yv[ps][w];
+        float tt = __fmul_rn(y, cr);  // rounded on its own, as the kernel's packed multiply
+        if (per_step) tt = fminf(fmaxf(tt, -7.0f), 7.0f);
+        float u = __fadd_rn(tt, rq::kMagic);
+        const float d = __fmaf_rn(__fadd_rn(u, -rq::kMagic), -1.0f, tt);
+        if (fabsf(d) >= rq::kTieBand || isinf(cr)) u = rq::exact_code(y, p.inv_sqrt_b, delta, cr, 7.0f, rq::kTieBand);
+        const uint32_t q8 = (__float_as_uint(u) & 0xFu) ^ 0x8u;
+        const int i = kk & 7;
+        s_act[(kk & ~7) + ((i & 1) ? 4 + (i >> 1) : (i >> 1))] = static_cast<uint8_t>(q8);
+        qs += q8;
+      }
+    }
+  }
+  const uint32_t wsum = __reduce_add_sync(0xffffffffu, qs);
+  if (lane == 0) s_wsum[warp] = wsum;
   __syncthreads();  // the operand bytes and code sums are complete
   return ok;
 }
 
 template <int kM, bool kGated, int kXB, typename OutT>
 __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
+  static_assert(kXB != 2 || kM == 1, "the one-launch linear takes one token");
   constexpr int kParts = kGated ? 2 : 1;  // 128-row weight groups per CTA
-  constexpr int kGvRing = gv_ring<kM, kGated>();
+  constexpr int kGvRing = gv_ring<kM, kGated, kXB>();
   constexpr int kActKb = kXB == 0 ? kBK / 2 : kBK;  // activation bytes per token and k-block
   __shared__ uint32_t s_part[kParts][128][kM];
   // split K: the slices of this CTA's rows from every CTA of the cluster, [source][row][part][m]
   __shared__ uint32_t s_recv[128 * kParts * kM];
   __shared__ __align__(8) uint64_t bar_recv;
-  // kXB 2: per token, the largest |rotated value| of this CTA's k-range and of every CTA's
-  // (received), the scale, and the sum of the offset codes q + 8 of this CTA's k-range
-  __shared__ uint32_t s_max[kM], s_maxes[8][kM], s_qsum[kM];
-  __shared__ float2 s_delta[kM];  // (scale, 1 / (scale sqrt(b)))
+  // kXB 2: the largest |rotated value| of each warp and of every CTA of the cluster (received),
+  // and each warp's sum of the offset codes q + 8 of this CTA's k-range
+  __shared__ uint32_t s_wmax[kGvThreads / 32], s_maxes[8], s_wsum[kGvThreads / 32];
   __shared__ __align__(8) uint64_t bar_max;
   // [kM][k-range] activation bytes of this CTA; kXB 2 then [kM][k-range] float rotated values
   // and one pass of C floats
@@ -278,7 +250,6 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
   const int R = 128 / S;  // rows this CTA finishes: [rank R, (rank + 1) R)
 
   for (int i = threadIdx.x; i < kParts * 128 * kM; i += kGvThreads) (&s_part[0][0][0])[i] = 0u;
-  if (kXB == 2 && threadIdx.x < kM) s_max[threadIdx.x] = s_qsum[threadIdx.x] = 0u;
   // kXB 2 with per-token scales: the CTAs of the cluster exchange their k-ranges' maxima
   // (unless one rotation pass is the whole row, which every CTA then rotates)
   const bool max_exchange = kXB == 2 && S > 1 && p.xscale == nullptr && p.K > p.C;
@@ -290,7 +261,7 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
       if (max_exchange) mbar_init(smem_u32(&bar_max), 1);
       mbar_init_fence();
       mbar_arrive_expect_tx(smem_u32(&bar_recv), static_cast<uint32_t>(S * R * kParts * kM * 4));
-      if (max_exchange) mbar_arrive_expect_tx(smem_u32(&bar_max), static_cast<uint32_t>(S * kM * 4));
+      if (max_exchange) mbar_arrive_expect_tx(smem_u32(&bar_max), static_cast<uint32_t>(S * 4));
     }
     cluster_arrive_relaxed();
   }
@@ -342,11 +313,12 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
   }
   bool landed = true, cluster_waited = false;
   if constexpr (kXB == 2) {
-    landed = rotate_quantize_range<kM>(p, static_cast<const OutT*>(p.x), kb0, kb1, rank, max_exchange, s_act, s_max,
-                                       s_maxes, s_qsum, s_delta, smem_u32(&bar_max));
+    float delta = 0.0f;
+    landed = rotate_quantize_token<OutT>(p, static_cast<const OutT*>(p.x), kb0, kb1, rank, max_exchange, s_act, s_wmax,
+                                         s_maxes, s_wsum, smem_u32(&bar_max), &delta);
     cluster_waited = max_exchange;
 #pragma unroll
-    for (int u = 0; u < kEnt; ++u) e_xs[u] = s_delta[min((threadIdx.x + u * kGvThreads) % kM, p.M - 1)].x;
+    for (int u = 0; u < kEnt; ++u) e_xs[u] = delta;
   } else {  // this CTA's k-range of every token's activation bytes, once, into shared memory
     const int row16 = (kb1 - kb0) * kActKb / 16;  // 16-byte pieces per token
     for (int i = threadIdx.x; i < p.M * row16; i += kGvThreads) {
@@ -437,8 +409,13 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
   __syncthreads();
   // kXB 2: 8 x the activation codes' sum over this CTA's k-range, taken out of its partials
   // (the sums of all ranks then hold S - 8 sum_k q_x, a signed value in 32-bit wrap-around)
-  auto xcorr = [&](int m) -> uint32_t {
-    if constexpr (kXB == 2) return 8u * s_qsum[m] - 64u * static_cast<uint32_t>((kb1 - kb0) * kBK);
+  uint32_t qsum = 0u;
+  if constexpr (kXB == 2) {
+#pragma unroll
+    for (int i = 0; i < kGvThreads / 32; ++i) qsum += s_wsum[i];
+  }
+  auto xcorr = [&](int) -> uint32_t {
+    if constexpr (kXB == 2) return 8u * qsum - 64u * static_cast<uint32_t>((kb1 - kb0) * kBK);
     return 0u;
   };
   if (S > 1) {
@@ -501,9 +478,9 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
 template <int kM, bool kGated, int kXB, typename OutT>
 cudaError_t launch_gv(const GemmArgs& a, GvParams p, int units) {
   auto kern = gemv_w4a4_kernel<kM, kGated, kXB, OutT>;
-  // the largest k-range of a CTA, for every token (kXB 2: and its rotated values, and one pass)
+  // the largest k-range of a CTA, for every token (kXB 2: and one rotation pass)
   size_t act = static_cast<size_t>(kM) * ((p.nkb + p.splits - 1) / p.splits) * (kXB == 0 ? kBK / 2 : kBK);
-  if (kXB == 2) act = 5 * act + 4 * static_cast<size_t>(p.C);
+  if (kXB == 2) act += 4 * static_cast<size_t>(p.C);
   if (act > static_cast<size_t>(kGemvActMax)) return kNotApplicable;
   if (act + 16 * 1024 > 48 * 1024) {  // with the static shared memory (up to 8.4 KB) past the default 48 KB
     cudaError_t e = prepare_kernel(reinterpret_cast<const void*>(kern), kGemvActMax);
@@ -588,18 +565,24 @@ cudaError_t launch_gemv_w4a4(const GemmArgs& a, bool* launched) {
   p.C = C;
   p.inv_sqrt_b = a.inv_sqrt_b;
   // one CTA per 128-row group (gated: per 128 hidden units, gate and up), K split over a cluster
-  // of up to 8 until the grid holds about two CTAs per SM
+  // of up to 8 until the grid holds about two CTAs per SM.  The one-launch linear (raw
+  // activations) doubles the split only while the grid holds at most 0.75 CTAs per SM, so a wide
+  // layer keeps about one CTA per SM with a deep weight ring and the next launch's CTAs fit beside
+  // it (measured on an 18-layer decode step: 455 us, against 540 us with the gate/up projection
+  // split in two and 472 us with its ring of four k-blocks).
   const int units = a.gated ? a.N / 256 : (a.N + 127) / 128;
   int splits = 1;
-  while (splits < 8 && 2 * splits <= p.nkb && units * splits < 2 * a.num_sms) splits *= 2;
-  p.splits = splits;
-  // raw activations: the CTAs' rotation and quantisation sit between the previous kernel and the
-  // weights' use.  Where the grid holds more than about 1.25 CTAs per SM and a CTA's weights do
-  // not all fit in the loads it issues before the wait, the rotate-quantise kernel ahead of the
-  // GEMV (its work overlapping the GEMV's first weight loads) measured faster.
   if (a.x_bytes == 3) {
-    const int ring = (a.gated ? gv_ring<1, true>() : gv_ring<1, false>()) * kGvPhases;
-    if (4 * units * splits > 5 * a.num_sms && (p.nkb + splits - 1) / splits >= ring) return cudaSuccess;
+    while (splits < 8 && 2 * splits <= p.nkb && 4 * units * splits <= 3 * a.num_sms) splits *= 2;
+  } else {
+    while (splits < 8 && 2 * splits <= p.nkb && units * splits < 2 * a.num_sms) splits *= 2;
+  }
+  p.splits = splits;
+  if (a.x_bytes == 3) {
+    for (int r = 0; r < splits; ++r) {  // a CTA holds the rotated values of at most kGvPasses passes
+      const int k0 = p.nkb * r / splits * kBK, k1 = p.nkb * (r + 1) / splits * kBK;
+      if ((k1 + C - 1) / C - k0 / C > kGvPasses) return cudaSuccess;
+    }
   }
   cudaError_t e;
   if (a.x_bytes == 3)

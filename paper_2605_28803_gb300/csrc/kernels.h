@@ -94,9 +94,9 @@ cudaError_t launch_gemm_fused(const GemmArgs& a, bool* launched);
 // enqueued) outside that range.  The outputs are those of launch_gemm_w4a4, bit for bit.
 // x_bytes 3 (M = 1): the raw activations x (dtype xdt == ydt, Hadamard block 2^log_b <= 2048
 // dividing the rotation pass) are rotated and quantised in the same launch; xscale is the step's
-// one scale or null for a per-token scale, xq and xsum are unused.  Taken only where the grid
-// holds at most about 1.25 CTAs per SM.  The outputs are those of the rotate-quantise kernel
-// followed by launch_gemm_w4a4, bit for bit.
+// one scale or null for a per-token scale, xq and xsum are unused.  Taken where each CTA's
+// k-range touches at most two rotation passes.  The outputs are those of the rotate-quantise
+// kernel followed by launch_gemm_w4a4, bit for bit.
 constexpr int kGemvMaxM = 4;
 cudaError_t launch_gemv_w4a4(const GemmArgs& a, bool* launched);
 

@@ -96,14 +96,15 @@ def test_one_launch_equals_two_launch_per_step(dt, K, N, had):
     layer.close()
 
 
-@pytest.mark.parametrize("K,N,had,M", [(4096, 256, 4096, 1), (2048, 2560, 2048, 2), (2048, 20480, 2048, 1)])
-def test_layers_outside_the_one_launch_take_two(K, N, had, M):
-    """A Hadamard block wider than one pass, more than one token, or a grid of more than about
-    1.25 CTAs per SM whose CTAs cannot load all their weights ahead of the previous kernel's end:
-    the two launches run (the workspace is written), with the same result."""
+@pytest.mark.parametrize("K,N,had,M,xdt", [(4096, 256, 4096, 1, "bf16"), (2048, 2560, 2048, 2, "bf16"),
+                                            (2048, 512, 2048, 1, "f32")])
+def test_layers_outside_the_one_launch_take_two(K, N, had, M, xdt):
+    """A Hadamard block wider than one pass, more than one token, or float32 input: the two
+    launches run (the workspace is written), with the same result."""
     rng = np.random.default_rng(K + N + M)
-    layer, _, _, _ = _layer(rng, N, K, had, "bf16", bias=False)
-    x = _input(rng, M, K, "bf16")
+    wcodes = rng.integers(-8, 8, (N, K)).astype(np.int8)
+    layer = G.make_layer(O.pack_int4(wcodes), np.full(N, 2 ** -8, np.float32), had, xdt, "bf16")
+    x = _input(rng, M, K, xdt)
     got, untouched = _one_launch(layer, x, -1, "bf16")
     assert not untouched
     assert np.array_equal(got, _two_launch(layer, x, -1, "bf16"))
