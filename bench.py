@@ -19,7 +19,8 @@ The line also carries the two layer stacks (skipped with --no-stacks):
          down 4096 -> 1024) at M = 50 tokens with per-step scale tables, one CUDA graph per
          denoising step: microseconds per step (L2 flushed before each) and per 10-step rollout;
   "backbone": 18 layers of hidden 2048 with the gated 16384 MLP, per-token scales, one forward
-         pass at M = 816 (TOPS) and at M = 1 (HBM-bound: GB/s of packed weights);
+         pass at M = 816 (TOPS) and at M = 1 (HBM-bound: GB/s of packed weights; one kernel
+         per linear);
   "dit"."w4a8" and "w4a8_gate_up": the W4A8 variant (8-bit activation codes) on the DiT stack
          and on the backbone's gate/up projection;
   "dit"."grouped": the DiT stack with Hadamard blocks of 64 and per-step, per-group tables.
@@ -637,7 +638,9 @@ def run_stacks(dev, stream, pk):
         st.close()
         del g, st
         torch.cuda.empty_cache()
-    bb["timing"] = "CUDA-graph replay of one forward (2 kernels per linear), L2 flushed before each"
+    bb["timing"] = ("CUDA-graph replay of one forward, L2 flushed before each; M = 816: the rotate-quantise "
+                    "kernel and the GEMM per linear; M = 1: one kernel per linear (the decode GEMV that "
+                    "rotates and quantises its token itself)")
     del scratch
     torch.cuda.empty_cache()
     return {"dit": dit, "backbone": bb, "w4a8_gate_up": w4a8_gu}
