@@ -89,7 +89,7 @@ template <typename XT>
 __device__ __forceinline__ bool rotate_quantize_token(const GvParams& p, const XT* __restrict__ x, int kb0, int kb1,
                                                       int rank, bool max_exchange, uint8_t* s_act, uint32_t* s_wmax,
                                                       uint32_t* s_maxes, uint32_t* s_wsum, uint32_t bar_max,
-                                                      float* delta_out) {
+                                                      bool hold, float* delta_out) {
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const int k0 = kb0 * kBK, range = (kb1 - kb0) * kBK;
   const int rmax = (p.nkb + p.splits - 1) / p.splits * kBK;  // the largest k-range of the cluster
@@ -181,7 +181,7 @@ __device__ __forceinline__ bool rotate_quantize_token(const GvParams& p, const X
   for (int i = 0; i < kGvThreads / 32; ++i) cmax = max(cmax, s_wmax[i]);
   if (max_exchange) {
     cluster_wait();  // pairs with the arrive at set-up: every CTA's barrier is initialised
-    if (t < p.splits)
+    if (t < p.splits && !hold)  // (test hook: held, no CTA sends anything; every receiving wait runs out)
       st_async_u32(mapa_shared(smem_u32(&s_maxes[rank]), static_cast<uint32_t>(t)), cmax,
                    mapa_shared(bar_max, static_cast<uint32_t>(t)));
     ok = mbar_wait_cluster(bar_max, 0) && ok;
@@ -242,6 +242,8 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int S = p.splits;
+  // test hook, read while the weights stream: held, the CTAs of a cluster send each other nothing
+  const bool hold = S > 1 && *const_cast<volatile int*>(&g_debug_hold_loads) != 0;
   const int unit = static_cast<int>(blockIdx.x) / S;
   const int rank = static_cast<int>(blockIdx.x) % S;  // the CTA's rank in its cluster of S
   const int kb0 = p.nkb * rank / S, kb1 = p.nkb * (rank + 1) / S;
@@ -315,7 +317,7 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
   if constexpr (kXB == 2) {
     float delta = 0.0f;
     landed = rotate_quantize_token<OutT>(p, static_cast<const OutT*>(p.x), kb0, kb1, rank, max_exchange, s_act, s_wmax,
-                                         s_maxes, s_wsum, smem_u32(&bar_max), &delta);
+                                         s_maxes, s_wsum, smem_u32(&bar_max), hold, &delta);
     cluster_waited = max_exchange;
 #pragma unroll
     for (int u = 0; u < kEnt; ++u) e_xs[u] = delta;
@@ -422,7 +424,8 @@ __global__ void __launch_bounds__(kGvThreads) gemv_w4a4_kernel(GvParams p) {
     if (!cluster_waited) cluster_wait();  // pairs with the arrive at set-up: every receive barrier is initialised
     // each partial goes to the CTA that finishes its row, as an asynchronous store completing on
     // that CTA's barrier; no CTA reads another's shared memory, so none waits for the others to leave
-    for (int i = threadIdx.x; i < 128 * kParts * kM; i += kGvThreads) {
+    // (test hook: held, nothing is sent and every CTA's wait runs out)
+    for (int i = threadIdx.x; i < (hold ? 0 : 128 * kParts * kM); i += kGvThreads) {
       const int row = i / (kParts * kM), part = (i / kM) % kParts, m = i % kM;
       const int d = row / R;
       const uint32_t dst = smem_u32(&s_recv[((rank * R + (row - d * R)) * kParts + part) * kM + m]);

@@ -48,3 +48,34 @@ def test_a_wait_that_runs_out_reports_timeout_and_the_next_launch_is_clean():
     y1, acc1 = G.gemm(layer, xq, xs, xsum)
     assert np.array_equal(acc1, acc0) and np.array_equal(y1, y0)
     layer.close()
+
+
+@pytest.mark.parametrize("M", [1, 2])
+def test_a_decode_gemv_wait_that_runs_out(M):
+    """The decode GEMV split over a cluster of CTAs: with the hook, no CTA sends its row maximum
+    (one launch, M = 1, K = 16384) or its partial sums (M = 1 and 2), so every receiving wait runs
+    out.  No asynchronous store is issued, so none is outstanding when the CTAs return.  The
+    kernel reports QVLA_ERR_TIMEOUT, writes nothing, and the next call is bit-exact."""
+    rng = np.random.default_rng(67 + M)
+    N, K = 2048, 16384
+    wcodes = rng.integers(-8, 8, (N, K)).astype(np.int8)
+    layer = G.make_layer(O.pack_int4(wcodes), np.full(N, 2 ** -9, np.float32), 2048, "bf16", "bf16")
+    x = torch.from_numpy(rng.standard_normal((M, K), dtype=np.float32)).to(torch.bfloat16)
+    y0 = G.linear(layer, x, ydt="bf16")
+    xg = x.to(G.DEV)
+    nbytes = Q.qvla_linear_workspace_bytes(layer, M)
+    work = torch.empty(nbytes, dtype=torch.uint8, device=G.DEV)
+    y = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device=G.DEV)
+    Q.qvla_check_device(G.stream())
+    Q.qvla_debug_set_hooks(20_000_000, True)
+    try:
+        Q.qvla_w4a4_linear(layer, xg, M, -1, y, work, nbytes, G.stream())
+        with pytest.raises(Q.QvlaError) as e:
+            Q.qvla_check_device(G.stream())
+        assert e.value.status == 6
+        assert torch.isnan(y).all().item()
+    finally:
+        Q.qvla_debug_set_hooks(0, False)
+    Q.qvla_check_device(G.stream())
+    assert np.array_equal(G.linear(layer, x, ydt="bf16"), y0)
+    layer.close()
