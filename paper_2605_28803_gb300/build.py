@@ -19,7 +19,7 @@ INCLUDE = os.path.join(os.path.dirname(PKG), "include")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 SOURCES = ["rotate_quant_f16.cu", "rotate_quant_bf16.cu", "rotate_quant_f32.cu", "rotate_quant_a8_f16.cu",
-           "rotate_quant_a8_bf16.cu", "rotate_quant_a8_f32.cu", "rotate_quant.cu", "a8_planes.cu", "block_rotate.cu", "gemm.cu", "gemm_fused.cu", "gemv.cu", "api.cu",
+           "rotate_quant_a8_bf16.cu", "rotate_quant_a8_f32.cu", "rotate_quant.cu", "rotate_quant_pass.cu", "a8_planes.cu", "block_rotate.cu", "gemm.cu", "gemm_fused.cu", "gemv.cu", "api.cu",
            "pack.cpp"]
 
 

@@ -949,16 +949,19 @@ qvla_status qvla_debug_set_hooks(unsigned long long wait_limit_ns, int hold_gemm
   QVLA_CUDA(qvla::set_debug_hooks_gemm(limit, hold), "test hooks (gemm)");
   QVLA_CUDA(qvla::set_debug_hooks_fused(limit, hold), "test hooks (fused)");
   QVLA_CUDA(qvla::set_debug_hooks_gemv(limit, hold), "test hooks (gemv)");
+  QVLA_CUDA(qvla::set_wait_limit_rqp(limit), "test hooks (rotate-quantise)");
   return QVLA_OK;
 }
 
 qvla_status qvla_check_device(void* stream) {
   g_last_error.clear();
-  unsigned int word = 0, word_fused = 0, word_gemv = 0;
+  unsigned int word = 0, word_fused = 0, word_gemv = 0, word_rqp = 0;
   QVLA_CUDA(qvla::read_and_clear_error_word(&word, static_cast<cudaStream_t>(stream)), "device check");
   QVLA_CUDA(qvla::read_and_clear_error_word_fused(&word_fused, static_cast<cudaStream_t>(stream)), "device check");
   QVLA_CUDA(qvla::read_and_clear_error_word_gemv(&word_gemv, static_cast<cudaStream_t>(stream)), "device check");
-  if ((word | word_fused | word_gemv) & 1u) return fail(QVLA_ERR_TIMEOUT, "a kernel wait ran out of its time limit");
+  QVLA_CUDA(qvla::read_and_clear_error_word_rqp(&word_rqp, static_cast<cudaStream_t>(stream)), "device check");
+  if ((word | word_fused | word_gemv | word_rqp) & 1u)
+    return fail(QVLA_ERR_TIMEOUT, "a kernel wait ran out of its time limit");
   return QVLA_OK;
 }
 

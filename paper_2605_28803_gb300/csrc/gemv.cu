@@ -37,14 +37,6 @@ __host__ __device__ constexpr int gv_ring() {
   return kM == 1 ? (kGated ? (kXB == 2 ? 6 : 2) : 4) : 2;
 }
 
-// Four bytes into the shared memory of a CTA of the cluster, completing 4 bytes of the
-// transaction count of that CTA's mbarrier (addresses from mapa_shared).
-__device__ __forceinline__ void st_async_u32(uint32_t cluster_addr, uint32_t v, uint32_t cluster_bar) {
-  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(cluster_addr), "r"(v),
-               "r"(cluster_bar)
-               : "memory");
-}
-
 struct GvParams {
   const uint8_t* wq;      // tiled weights [groups][K/128][128][64 B]
   const uint8_t* xq;      // activations: operand bytes [M][K] (kXB 1) or packed nibbles [M][K/2] (kXB 0)

@@ -32,6 +32,14 @@ struct RotQuantArgs {
   cudaStream_t stream;
 };
 bool rotate_quant_supported(int log_b);
+// The rotate-quantise kernel in passes (rotate_quant_pass.cu): up to 8 rows of 16-bit
+// activations into operand bytes (out_mode 1) with one scale per row, per token or per step,
+// Hadamard block <= 2048 and at most 8 passes of 2048 (or fewer, smaller) channels per row.
+// *launched is false (nothing enqueued) outside that range; the outputs are those of the
+// row-per-warp kernel, bit for bit.  launch_rotate_quant takes it first.
+cudaError_t launch_rotate_quant_pass(const RotQuantArgs& a, bool* launched);
+cudaError_t read_and_clear_error_word_rqp(unsigned int* out, cudaStream_t stream);
+cudaError_t set_wait_limit_rqp(unsigned long long wait_limit_ns);
 cudaError_t launch_rotate_quant(const RotQuantArgs& a);
 
 // ---- int8 codes to the W4A8 GEMM's operand planes (a8_planes.cu) ----

@@ -153,6 +153,13 @@ __device__ __forceinline__ void st_async_v4(uint32_t cluster_addr, float4 v, uin
                : "memory");
 }
 // The address of the same shared-memory variable in CTA `rank` of the cluster.
+// Four bytes into the shared memory of a CTA of the cluster, completing 4 bytes of the
+// transaction count of that CTA's mbarrier (addresses from mapa_shared).
+__device__ __forceinline__ void st_async_u32(uint32_t cluster_addr, uint32_t v, uint32_t cluster_bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(cluster_addr), "r"(v),
+               "r"(cluster_bar)
+               : "memory");
+}
 __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
   uint32_t r;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
