@@ -32,7 +32,7 @@ struct RotQuantArgs {
   cudaStream_t stream;
 };
 bool rotate_quant_supported(int log_b);
-// The rotate-quantise kernel in passes (rotate_quant_pass.cu): up to 8 rows of 16-bit
+// The rotate-quantise kernel in passes (rotate_quant_pass.cu): up to 64 rows of 16-bit
 // activations into operand bytes (out_mode 1) with one scale per row, per token or per step,
 // Hadamard block <= 2048 and at most 8 passes of 2048 (or fewer, smaller) channels per row.
 // *launched is false (nothing enqueued) outside that range; the outputs are those of the

@@ -24,7 +24,7 @@ namespace {
 
 constexpr int kRqpThreads = 256;
 constexpr int kRqpMaxPasses = 8;  // a cluster of at most 8 CTAs (K <= 16384)
-constexpr int kRqpMaxRows = 8;    // the rows it takes (more rows go to the row-per-warp kernel)
+constexpr int kRqpMaxRows = 64;   // the rows it takes (more rows go to the row-per-warp kernel)
 
 struct RqpParams {
   const void* x;            // [M][K] activations
@@ -219,9 +219,10 @@ cudaError_t launch_rqp(const RotQuantArgs& a, const RqpParams& p) {
 cudaError_t launch_rotate_quant_pass(const RotQuantArgs& a, bool* launched) {
   *launched = false;
   // 16-bit activations into 4-bit operand bytes, one scale per row (per token or per step), for
-  // a few rows: there the latency of one row decides, and a pass's 256 threads cut it (measured,
-  // one call: 1 x 2048 6.8 against 8.8 us, 4 x 16384 8.8 against 10.9 us).  At hundreds of rows
-  // the row-per-warp kernel's cheaper stages per element win (816 x 16384: 27.3 against 41.6 us).
+  // up to 64 rows: there the latency of one row decides, and a pass's 256 threads cut it
+  // (measured, one call: 1 x 2048 6.8 against 8.8 us, 4 x 16384 8.8 against 10.9 us; the DiT
+  // step at 50 tokens 691 -> 647 us).  At hundreds of rows the row-per-warp kernel's cheaper
+  // stages per element win (816 x 16384: 27.3 against 41.6 us).
   if (a.out_mode != 1 || (a.mode != 0 && a.mode != 1) || (a.xdt != 0 && a.xdt != 1) || a.gshift < 30 ||
       a.xgsum != nullptr || a.M < 1 || a.M > kRqpMaxRows)
     return cudaSuccess;

@@ -3,7 +3,7 @@ activations into the GEMM's operand bytes, one CTA per pass of up to 2048 channe
 a row in a cluster that exchanges the row maximum and gathers the code sum (Sec. 4.1 Eq. 3-5,
 Sec. 4.2 Eq. 5-6).
 
-qvla_linear_quantize takes it for f16/bf16 layers at up to 8 rows; its codes, scales and code
+qvla_linear_quantize takes it for f16/bf16 layers at up to 64 rows; its codes, scales and code
 sums must be the bits of the row-per-warp kernel, which the packed-code entry
 qvla_rotate_quantize_rows still runs (and which tests/test_gpu_rotate_quant.py pins to the
 oracle).  Shapes cover one to eight passes per row, passes of 128 to 2048 channels, Hadamard
@@ -71,8 +71,8 @@ def _input(M, K, seed, dt):
     return W.as_dtype(x, dt)
 
 
-SHAPES = [(8, 2048, 2048), (4, 16384, 2048), (1, 1024, 1024), (3, 3072, 1024), (7, 384, 128), (2, 4096, 64),
-          (5, 16384, 512), (5, 2048, 1), (1, 128, 128), (6, 640, 128)]
+SHAPES = [(64, 2048, 2048), (4, 16384, 2048), (50, 1024, 1024), (3, 3072, 1024), (7, 384, 128), (33, 4096, 64),
+          (5, 16384, 512), (5, 2048, 1), (1, 128, 128), (6, 640, 128), (50, 4096, 1024)]
 
 
 @pytest.mark.parametrize("dt", ["f16", "bf16"])
@@ -118,7 +118,7 @@ def test_pass_kernel_exact_ties(K):
     assert np.all(q1[1, :K - 3] == 0) and q1[1, K - 3] == 7
 
 
-@pytest.mark.parametrize("M,K,had", [(8, 16384, 2048), (4, 2048, 2048)])
+@pytest.mark.parametrize("M,K,had", [(64, 16384, 2048), (4, 2048, 2048)])
 def test_pass_kernel_against_oracle(M, K, had):
     x = _input(M, K, 7 + M, "bf16")
     q1, s1, c1 = _pass_kernel(x, had)
