@@ -731,8 +731,9 @@ SWEEP_KN = ((1024, 1024), (1024, 4096), (2048, 2048), (2048, 16384), (16384, 204
 
 def run_sweep(dev, stream, pk, oracle_point=True, points_only=None):
     """The single-linear sweep: qvla_w4a4_linear at M in SWEEP_M x (K, N) in SWEEP_KN, f16 in and
-    out, per-token scales, Hadamard K (2048 blocks at K = 16384).  Each point: 10 calls, L2
-    flushed before each, CUDA events around the rotate + quantise and the GEMM launches.  The
+    out, per-token scales, Hadamard K (2048 blocks at K = 16384).  Each point: 10 calls of the
+    linear, L2 flushed before each, CUDA events around it; then 10 calls of its two halves
+    (qvla_linear_quantize, qvla_linear_gemm) with events around each.  The
     weights are uniform random code bytes (the time of a linear does not depend on its values);
     the activations are drawn on the device (N(0,1), 0.5% channels x20)."""
     from paper_2605_28803_gb300 import qvla as Q
@@ -757,7 +758,7 @@ def run_sweep(dev, stream, pk, oracle_point=True, points_only=None):
         for m in ms:
             xm, ym = x[:m], y[:m]
 
-            def call(ev=None):
+            def halves(ev=None):
                 if ev:
                     ev[0].record(stream)
                 Q.qvla_linear_quantize(layer, xm, m, -1, work, nb, stream)
@@ -767,23 +768,41 @@ def run_sweep(dev, stream, pk, oracle_point=True, points_only=None):
                 if ev:
                     ev[2].record(stream)
 
-            for _ in range(3):
-                call()
+            def linear(ev=None):
+                if ev:
+                    ev[0].record(stream)
+                Q.qvla_w4a4_linear(layer, xm, m, -1, ym, work, nb, stream)
+                if ev:
+                    ev[1].record(stream)
+
+            def timed(fn, nev):
+                for _ in range(3):
+                    fn()
+                torch.cuda.synchronize()
+                evs = []
+                for _ in range(10):
+                    scratch.zero_()
+                    e = [torch.cuda.Event(enable_timing=True) for _ in range(nev)]
+                    fn(e)
+                    evs.append(e)
+                torch.cuda.synchronize()
+                return evs
+
+            # launches of the whole linear: one where the decode GEMV rotates and quantises
+            # itself (the workspace then stays untouched), else the two halves
+            work.fill_(0xA5)
+            linear()
             torch.cuda.synchronize()
-            evs = []
-            for _ in range(10):
-                scratch.zero_()
-                e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-                call(e)
-                evs.append(e)
-            torch.cuda.synchronize()
-            t_all = statistics.median(e[0].elapsed_time(e[2]) for e in evs) * 1e-3
-            t_rq = statistics.median(e[0].elapsed_time(e[1]) for e in evs) * 1e-3
-            t_gemm = statistics.median(e[1].elapsed_time(e[2]) for e in evs) * 1e-3
+            launches = 1 if bool(torch.all(work == 0xA5).item()) else 2
+            ev_l = timed(linear, 2)
+            ev_h = timed(halves, 3)
+            t_all = statistics.median(e[0].elapsed_time(e[1]) for e in ev_l) * 1e-3
+            t_rq = statistics.median(e[0].elapsed_time(e[1]) for e in ev_h) * 1e-3
+            t_gemm = statistics.median(e[1].elapsed_time(e[2]) for e in ev_h) * 1e-3
             ops, nbytes = 2 * m * n * k, _linear_bytes(m, k, n)
-            pt = {"M": m, "K": k, "N": n, "us": round(t_all * 1e6, 2), "us_rotate_quantize": round(t_rq * 1e6, 2),
-                  "us_gemm": round(t_gemm * 1e6, 2), "tops": round(ops / t_all / 1e12, 2),
-                  "gbs": round(nbytes / t_all / 1e9, 1)}
+            pt = {"M": m, "K": k, "N": n, "us": round(t_all * 1e6, 2), "launches": launches,
+                  "us_rotate_quantize": round(t_rq * 1e6, 2), "us_gemm": round(t_gemm * 1e6, 2),
+                  "tops": round(ops / t_all / 1e12, 2), "gbs": round(nbytes / t_all / 1e9, 1)}
             pt["roofline"] = _roofline_point(ops, nbytes, t_all, pk)
             points.append(pt)
         Q.qvla_check_device(stream)
@@ -793,8 +812,10 @@ def run_sweep(dev, stream, pk, oracle_point=True, points_only=None):
     del scratch
     torch.cuda.empty_cache()
     out = {"points": points,
-           "timing": "median of 10 calls of qvla_w4a4_linear's two halves, L2 flushed (256 MB write) before each; "
-                     "bytes = 2MK + NK/2 + 4N + 2MN; roofline = HBM left of the ridge, burst E4M3 right of it",
+           "timing": "us: median of 10 calls of qvla_w4a4_linear (launches: 1 where the decode GEMV takes the "
+                     "token, else 2), L2 flushed (256 MB write) before each; us_rotate_quantize / us_gemm: the "
+                     "two halves called separately, likewise; bytes = 2MK + NK/2 + 4N + 2MN; roofline = HBM left "
+                     "of the ridge, burst E4M3 right of it",
            "ridge_ops_per_byte": round(pk["tflops"] * 1e12 / (pk["gbs"] * 1e9), 1)}
     if oracle_point:
         out["oracle_point"] = _oracle_sweep_point()
