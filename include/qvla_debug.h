@@ -21,8 +21,9 @@ extern "C" {
  *                   records QVLA_ERR_TIMEOUT (read by qvla_check_device), issues no MMA, leaves
  *                   y unwritten and returns.  The decode GEMV (one to four tokens, K split over a
  *                   cluster) then sends nothing between its CTAs (no row maximum, no partial
- *                   sum), so their receiving waits run out the same way.  0 restores normal
- *                   operation.
+ *                   sum), and neither do the passes of a row in the few-row rotate-quantise
+ *                   kernel (no row maximum, no code sum), so their receiving waits run out the
+ *                   same way.  0 restores normal operation.
  * Synchronises the device first; affects every later launch on the current device until called
  * again. */
 qvla_status qvla_debug_set_hooks(unsigned long long wait_limit_ns, int hold_gemm_loads);

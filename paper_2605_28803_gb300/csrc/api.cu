@@ -949,7 +949,7 @@ qvla_status qvla_debug_set_hooks(unsigned long long wait_limit_ns, int hold_gemm
   QVLA_CUDA(qvla::set_debug_hooks_gemm(limit, hold), "test hooks (gemm)");
   QVLA_CUDA(qvla::set_debug_hooks_fused(limit, hold), "test hooks (fused)");
   QVLA_CUDA(qvla::set_debug_hooks_gemv(limit, hold), "test hooks (gemv)");
-  QVLA_CUDA(qvla::set_wait_limit_rqp(limit), "test hooks (rotate-quantise)");
+  QVLA_CUDA(qvla::set_debug_hooks_rqp(limit, hold), "test hooks (rotate-quantise)");
   return QVLA_OK;
 }
 

@@ -39,7 +39,7 @@ bool rotate_quant_supported(int log_b);
 // row-per-warp kernel, bit for bit.  launch_rotate_quant takes it first.
 cudaError_t launch_rotate_quant_pass(const RotQuantArgs& a, bool* launched);
 cudaError_t read_and_clear_error_word_rqp(unsigned int* out, cudaStream_t stream);
-cudaError_t set_wait_limit_rqp(unsigned long long wait_limit_ns);
+cudaError_t set_debug_hooks_rqp(unsigned long long wait_limit_ns, int hold);
 cudaError_t launch_rotate_quant(const RotQuantArgs& a);
 
 // ---- int8 codes to the W4A8 GEMM's operand planes (a8_planes.cu) ----

@@ -23,6 +23,9 @@ namespace qvla {
 namespace {
 
 constexpr int kRqpThreads = 256;
+// test hook (qvla_debug.h): nonzero, the CTAs of a cluster send each other nothing, so every
+// receiving wait runs out
+static __device__ int g_rqp_hold;
 constexpr int kRqpMaxPasses = 8;  // a cluster of at most 8 CTAs (K <= 16384)
 constexpr int kRqpMaxRows = 64;   // the rows it takes (more rows go to the row-per-warp kernel)
 
@@ -48,6 +51,7 @@ __global__ void __launch_bounds__(kRqpThreads) rotate_quant_pass_kernel(RqpParam
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const int m = static_cast<int>(blockIdx.x) / P, rank = static_cast<int>(blockIdx.x) % P;
   const bool exch_max = !kStep && P > 1;
+  const bool hold = P > 1 && *const_cast<volatile int*>(&g_rqp_hold) != 0;
   if (P > 1) {
     // the cluster barrier completed before the first send guarantees every receiver's barrier
     if (t == 0) {
@@ -136,7 +140,7 @@ __global__ void __launch_bounds__(kRqpThreads) rotate_quant_pass_kernel(RqpParam
   bool ok = true;
   if (P > 1) cluster_wait();  // pairs with the arrive at set-up
   if (exch_max) {
-    if (t < P)
+    if (t < P && !hold)
       st_async_u32(mapa_shared(smem_u32(&s_maxes[rank]), static_cast<uint32_t>(t)), cmax,
                    mapa_shared(smem_u32(&bar_max), static_cast<uint32_t>(t)));
     ok = mbar_wait_cluster(smem_u32(&bar_max), 0);
@@ -177,7 +181,7 @@ __global__ void __launch_bounds__(kRqpThreads) rotate_quant_pass_kernel(RqpParam
 #pragma unroll
   for (int i = 0; i < kRqpThreads / 32; ++i) csum += s_wsum[i];
   if (P > 1) {
-    if (t == 0)
+    if (t == 0 && !hold)
       st_async_u32(mapa_shared(smem_u32(&s_sums[rank]), 0u), csum, mapa_shared(smem_u32(&bar_sum), 0u));
     if (rank == 0) {
       ok = mbar_wait_cluster(smem_u32(&bar_sum), 0) && ok;
@@ -260,11 +264,13 @@ cudaError_t read_and_clear_error_word_rqp(unsigned int* out, cudaStream_t stream
   return cudaMemcpyToSymbol(g_error_word, &zero, sizeof(unsigned int));
 }
 
-cudaError_t set_wait_limit_rqp(unsigned long long wait_limit_ns) {
+cudaError_t set_debug_hooks_rqp(unsigned long long wait_limit_ns, int hold) {
   const unsigned long long v = wait_limit_ns ? wait_limit_ns : kWaitLimitNs;
   cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return e;
-  return cudaMemcpyToSymbol(g_wait_limit_ns, &v, sizeof(v));
+  e = cudaMemcpyToSymbol(g_wait_limit_ns, &v, sizeof(v));
+  if (e != cudaSuccess) return e;
+  return cudaMemcpyToSymbol(g_rqp_hold, &hold, sizeof(hold));
 }
 
 }  // namespace qvla

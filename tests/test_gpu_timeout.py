@@ -79,3 +79,32 @@ def test_a_decode_gemv_wait_that_runs_out(M):
     Q.qvla_check_device(G.stream())
     assert np.array_equal(G.linear(layer, x, ydt="bf16"), y0)
     layer.close()
+
+
+def test_a_rotate_quantize_pass_wait_that_runs_out():
+    """The few-row rotate-quantise kernel with a row of 8 passes in a cluster: with the hook, no pass
+    sends its maximum or its code sum, so the waits run out; the launch reports QVLA_ERR_TIMEOUT
+    and returns with no asynchronous store outstanding, and the next call is bit-exact."""
+    rng = np.random.default_rng(71)
+    M, K = 2, 16384
+    layer = G.make_layer(np.zeros((16, K // 2), np.uint8), np.ones(16, np.float32), 2048, "bf16", "bf16")
+    x = torch.from_numpy(rng.standard_normal((M, K), dtype=np.float32)).to(torch.bfloat16).to(G.DEV)
+    nbytes = Q.qvla_linear_workspace_bytes(layer, M)
+    ref = torch.zeros(nbytes, dtype=torch.uint8, device=G.DEV)
+    Q.qvla_linear_quantize(layer, x, M, -1, ref, nbytes, G.stream())
+    Q.qvla_check_device(G.stream())
+    work = torch.zeros(nbytes, dtype=torch.uint8, device=G.DEV)
+    Q.qvla_debug_set_hooks(20_000_000, True)
+    try:
+        Q.qvla_linear_quantize(layer, x, M, -1, work, nbytes, G.stream())
+        with pytest.raises(Q.QvlaError) as e:
+            Q.qvla_check_device(G.stream())
+        assert e.value.status == 6
+    finally:
+        Q.qvla_debug_set_hooks(0, False)
+    Q.qvla_check_device(G.stream())
+    work.zero_()
+    Q.qvla_linear_quantize(layer, x, M, -1, work, nbytes, G.stream())
+    Q.qvla_check_device(G.stream())
+    assert torch.equal(work, ref)  # codes, scales and sums (the padding is zero in both)
+    layer.close()
