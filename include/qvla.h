@@ -250,10 +250,14 @@ qvla_status qvla_rotated_absmax_groups(const void* x, qvla_dtype xdt, int M, int
 qvla_status qvla_gemm_w4a4(const qvla_layer* layer, const uint8_t* xq, const float* xscale,
                            const int32_t* xsum, int M, void* y, int32_t* acc, void* stream);
 
-/* Bytes of device workspace qvla_w4a4_linear needs for M rows (a multiple of 256): the codes
+/* Bytes of device workspace qvla_w4a4_linear takes for M rows (a multiple of 256): the codes
  * travel between its two kernels as one tensor-core operand byte each (M x K bytes), plus the
  * scales, the code sums and the per-group code sums (M x G x 4 bytes), and, for a layer with an
- * online rotation, x . P . BlockDiag(U_b) (M x K elements of the activation dtype). */
+ * online rotation, x . P . BlockDiag(U_b) (M x K elements of the activation dtype).  Where the
+ * GEMM's tiles could leave SMs idle (M > 128, not gated, fewer 128 x 256 tiles than SMs) it adds
+ * room for splitting each tile's K into up to 4 work units: 4 FP32 partials per output (M and N
+ * rounded up to 256) and 4 bytes of counter per 128 x 128 tile.  The linear also runs in a
+ * workspace of the first parts only; its GEMM then does not split K. */
 size_t qvla_linear_workspace_bytes(const qvla_layer* layer, int M);
 
 /* The whole online linear (Sec. 4): rotate + quantise x (as qvla_rotate_quantize, step as

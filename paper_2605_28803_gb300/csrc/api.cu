@@ -107,7 +107,7 @@ qvla_status check_rows(int M) {
 
 qvla_status launch_rq(const void* x, int xdt, int M, int K, int had_block, int mode, const float* step_scale,
                       uint8_t* xq, float* xscale, int32_t* xsum, float* absmax, void* stream, int out_mode = 0,
-                      int group = 0, int32_t* xgsum = nullptr) {
+                      int group = 0, int32_t* xgsum = nullptr, int32_t* zero = nullptr, int zero_n = 0) {
   qvla::RotQuantArgs a;
   a.x = x;
   a.xdt = xdt;
@@ -124,6 +124,8 @@ qvla_status launch_rq(const void* x, int xdt, int M, int K, int had_block, int m
   a.out_mode = out_mode;
   a.gshift = group > 0 ? ilog2_exact(group) : 30;
   a.xgsum = xgsum;
+  a.zero = zero;
+  a.zero_n = zero_n;
   a.stream = static_cast<cudaStream_t>(stream);
   QVLA_CUDA(qvla::launch_rotate_quant(a), "rotate_quantize launch");
   return QVLA_OK;
@@ -578,9 +580,17 @@ qvla_status qvla_rotate_quantize_rows_a8(const void* x, qvla_dtype xdt, int M, i
 }  // extern "C"
 
 namespace {
+// The workspace's room for the GEMM's split of K: the work units' partials and the tiles' counters.
+struct PartWorkspace {
+  float* ws = nullptr;
+  size_t floats = 0;
+  int32_t* cnt = nullptr;
+  int n = 0;
+};
+
 qvla_status launch_gemm(const qvla_layer* L, const uint8_t* xq, int x_bytes, const float* xscale, const int32_t* xsum,
                         int M, void* y, int32_t* acc, void* stream, const float* gscale = nullptr,
-                        const int32_t* xgsum = nullptr) {
+                        const int32_t* xgsum = nullptr, const PartWorkspace* pw = nullptr) {
   qvla::GemmArgs a;
   a.xq = xq;
   a.x_bytes = x_bytes;
@@ -603,6 +613,12 @@ qvla_status launch_gemm(const qvla_layer* L, const uint8_t* xq, int x_bytes, con
     a.wgcorr = L->wgcorr;
     a.group = L->group;
   }
+  if (pw != nullptr && pw->ws != nullptr) {
+    a.part_ws = pw->ws;
+    a.part_ws_floats = pw->floats;
+    a.part_cnt = pw->cnt;
+    a.part_cnt_n = pw->n;
+  }
   a.num_sms = num_sms(L->device);
   a.stream = static_cast<cudaStream_t>(stream);
   QVLA_CUDA(qvla::launch_gemm_w4a4(a), "gemm launch");
@@ -624,12 +640,35 @@ qvla_status qvla_gemm_w4a4(const qvla_layer* L, const uint8_t* xq, const float* 
   return launch_gemm(L, xq, 0, xscale, xsum, M, y, acc, stream);
 }
 
-size_t qvla_linear_workspace_bytes(const qvla_layer* L, int M) {
-  if (!L || M <= 0) return 0;
+namespace {
+// The linear's workspace: what it needs, and the optional room for the GEMM's split of K.
+size_t workspace_min(const qvla_layer* L, int M) {
   // the codes travel between the two kernels as one operand byte each; then the scales, the
   // code sums and the per-group code sums (used with per-group step scales)
   return round256(static_cast<size_t>(M) * L->K) + round256(static_cast<size_t>(M) * 4) * 2 +
          round256(static_cast<size_t>(M) * L->G * 4) + (L->rblock ? round256(rotated_bytes(L, M)) : 0);
+}
+constexpr int kMaxParts = 4;  // work units per tile of the GEMM's split of K
+// The GEMM's split of K: a non-gated token-major layer (M > 128) whose 128 x 256 tiles leave SMs
+// idle may split; room for kMaxParts FP32 partials of every output (rows and weight rows padded to
+// 256) and a count for each 128 x 128 tile covers every tile shape it can take.
+bool may_split(const qvla_layer* L, int M) {
+  if (M <= 128 || L->gated) return false;
+  return static_cast<long>((M + 127) / 128) * ((L->N + 255) / 256) < num_sms(L->device);
+}
+size_t split_floats(const qvla_layer* L, int M) {
+  return static_cast<size_t>((M + 255) / 256) * 256 * ((L->N + 255) / 256) * 256 * kMaxParts;
+}
+int split_counts(const qvla_layer* L, int M) { return ((M + 127) / 128) * ((L->N + 127) / 128); }
+size_t workspace_parts(const qvla_layer* L, int M) {
+  if (!may_split(L, M)) return 0;
+  return round256(split_floats(L, M) * 4) + round256(static_cast<size_t>(split_counts(L, M)) * 4);
+}
+}  // namespace
+
+size_t qvla_linear_workspace_bytes(const qvla_layer* L, int M) {
+  if (!L || M <= 0) return 0;
+  return workspace_min(L, M) + workspace_parts(L, M);
 }
 
 namespace {
@@ -639,12 +678,13 @@ struct LinearWorkspace {
   int32_t* xsum;     // [M]
   int32_t* xgsum;    // [M][G]
   void* xrot;        // [M][K] x . P . BlockDiag(U_b) in the activation dtype (layers with an online rotation)
+  PartWorkspace parts;  // the GEMM's split of K (empty when the workspace has no room for it)
 };
 
 qvla_status carve_workspace(const qvla_layer* L, int M, void* workspace, size_t workspace_bytes, LinearWorkspace* w) {
   if (!workspace) return fail(QVLA_ERR_INVALID_ARG, "workspace must not be NULL");
   if (reinterpret_cast<uintptr_t>(workspace) & 255u) return fail(QVLA_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
-  const size_t need = qvla_linear_workspace_bytes(L, M);
+  const size_t need = workspace_min(L, M);
   if (workspace_bytes < need)
     return fail(QVLA_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed", workspace_bytes, need);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
@@ -653,6 +693,13 @@ qvla_status carve_workspace(const qvla_layer* L, int M, void* workspace, size_t 
   w->xsum = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(w->xscale) + round256(static_cast<size_t>(M) * 4));
   w->xgsum = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(w->xsum) + round256(static_cast<size_t>(M) * 4));
   w->xrot = reinterpret_cast<uint8_t*>(w->xgsum) + round256(static_cast<size_t>(M) * L->G * 4);
+  const size_t parts = workspace_parts(L, M);
+  if (parts > 0 && workspace_bytes >= need + parts) {  // room for the GEMM's split of K
+    w->parts.ws = reinterpret_cast<float*>(ws + need);
+    w->parts.floats = split_floats(L, M);
+    w->parts.cnt = reinterpret_cast<int32_t*>(ws + need + round256(w->parts.floats * 4));
+    w->parts.n = split_counts(L, M);
+  }
   return QVLA_OK;
 }
 
@@ -686,7 +733,9 @@ qvla_status qvla_linear_quantize(const qvla_layer* L, const void* x, int M, int 
   if (qvla_status s = carve_workspace(L, M, workspace, workspace_bytes, &w)) return s;
   const void* xin = nullptr;
   if (qvla_status s = online_input(L, x, M, w, stream, &xin)) return s;
-  return launch_rq(xin, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr, stream, 1);
+  // (the rotate-quantise kernel also clears the GEMM's counters of the split of K)
+  return launch_rq(xin, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr, stream, 1, 0,
+                   nullptr, w.parts.cnt, w.parts.n);
 }
 
 qvla_status qvla_linear_gemm(const qvla_layer* L, const void* workspace, size_t workspace_bytes, int M, void* y,
@@ -699,7 +748,7 @@ qvla_status qvla_linear_gemm(const qvla_layer* L, const void* workspace, size_t 
   if (!aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "y must be 16-byte aligned");
   LinearWorkspace w;
   if (qvla_status s = carve_workspace(L, M, const_cast<void*>(workspace), workspace_bytes, &w)) return s;
-  return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream);
+  return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream, nullptr, nullptr, &w.parts);
 }
 
 namespace {
@@ -818,9 +867,9 @@ qvla_status qvla_w4a4_linear(const qvla_layer* L, const void* x, int M, int step
     return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream, ss, w.xgsum);
   }
   if (qvla_status s = launch_rq(xin, L->xdt, M, L->K, L->had_block, ss ? 1 : 0, ss, w.xb, w.xscale, w.xsum, nullptr,
-                                stream, 1))
+                                stream, 1, 0, nullptr, w.parts.cnt, w.parts.n))
     return s;
-  return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream);
+  return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream, nullptr, nullptr, &w.parts);
 }
 
 }  // extern "C"
@@ -932,7 +981,8 @@ qvla_status qvla_w4a4_linear_noalloc(const qvla_layer* L, const void* x, int M, 
   if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
   if (qvla_status s = check_layer_device(L)) return s;  // the scratch looked up is the current device's
   if (qvla_status s = check_rows(M)) return s;
-  const size_t need = qvla_linear_workspace_bytes(L, M);
+  // the scratch holds what the linear needs; the GEMM's split of K runs only where it fits as well
+  const size_t need = workspace_min(L, M);
   if (need > QVLA_NOALLOC_SCRATCH_BYTES)
     return fail(QVLA_ERR_UNSUPPORTED, "M=%d, K=%d needs %zu bytes of scratch; the allocation-free linear holds %zu", M, L->K,
                 need, static_cast<size_t>(QVLA_NOALLOC_SCRATCH_BYTES));

@@ -24,29 +24,54 @@ cudaError_t launch_grouped(const GemmArgs& a) {
 // (2000 + 344 / k-block) and 2000 + waves x (2500 + 560 / k-block); CTA pairs (256 tokens over two
 // SMs, half the weight rows staged per SM) 3900 + waves x (1000 + 351 / k-block) and 3800 + waves
 // x (2900 + 375 / k-block).  A pair wave holds half as many tiles, each of twice the tokens.
+// A non-gated layer whose tiles leave SMs (or pairs) idle may split each tile's k-blocks into 2
+// or 4 work units of at least 16 k-blocks (their partials in the caller's workspace, the tile's
+// last unit finishing it): a wave of units then costs per_tile + split + k-blocks per unit x
+// per_kb, with split fitted on 816 x 16384 -> 2048: 4900 ns for single CTAs (128-wide tiles in 4
+// parts, 56.0 us against 53.9 whole) and 14500 for pairs (256-wide tiles in 2 parts, 45.2 us).
 enum class TileShape { kSingle128, kSingle256, kPair128, kPair256 };
 
-TileShape token_major_shape(const GemmArgs& a) {
+TileShape token_major_shape(const GemmArgs& a, int* parts) {
   const long nkb = a.K / kBK, sms = a.num_sms, npairs = a.num_sms / 2;
   const long t1 = (a.M + kBM - 1) / kBM, t2 = (a.M + 2 * kBM - 1) / (2 * kBM);
   const long n128 = a.gated ? 0 : (a.N + 127) / 128, n256 = (a.N + 255) / 256;
-  auto est = [nkb](long tiles, long units, long fixed, long per_tile, long per_kb) {
-    return fixed + (tiles + units - 1) / units * (per_tile + nkb * per_kb);
+  const bool can_split = !a.gated && a.part_ws != nullptr && a.part_cnt != nullptr;
+  // estimated time of a shape (tiles of bn weight rows, `halves` CTAs each) at its best split
+  auto est = [&](long tiles, long units, long fixed, long per_tile, long per_kb, long bn, long halves, int* q_out) {
+    const long split = halves == 2 ? 14500 : 4900;
+    const long whole = fixed + (tiles + units - 1) / units * (per_tile + nkb * per_kb);
+    long best = whole;
+    *q_out = 1;
+    if (!can_split || tiles >= units) return best;
+    for (int q = 2; q <= 4; q *= 2) {
+      if (nkb / q < 16 || static_cast<size_t>(tiles * halves * q * kBM * bn) > a.part_ws_floats ||
+          tiles * halves > a.part_cnt_n)
+        continue;
+      const long t = fixed + (tiles * q + units - 1) / units * (per_tile + split + (nkb + q - 1) / q * per_kb);
+      if (t < best && 10 * t < 9 * whole) {  // a split only where it is estimated 10% faster
+        best = t;
+        *q_out = q;
+      }
+    }
+    return best;
   };
+  int q = 1;
   TileShape best = TileShape::kSingle256;
-  long t = est(t1 * n256, sms, 2000, 2500, 560);
+  long t = est(t1 * n256, sms, 2000, 2500, 560, 256, 1, &q);
+  *parts = q;
   auto consider = [&](TileShape s, long v) {
     if (v < t) {
       t = v;
       best = s;
+      *parts = q;
     }
   };
-  if (n128) consider(TileShape::kSingle128, est(t1 * n128, sms, 2300, 2000, 344));
+  if (n128) consider(TileShape::kSingle128, est(t1 * n128, sms, 2300, 2000, 344, 128, 1, &q));
   // pairs need a few k-blocks per tile to hide their larger per-tile hand-over (measured at
   // K = 256: 12% slower than single CTAs where this estimate favoured the pair)
   if (a.M > kBM && npairs > 0 && nkb >= 8) {
-    consider(TileShape::kPair256, est(t2 * n256, npairs, 3800, 2900, 375));
-    if (n128) consider(TileShape::kPair128, est(t2 * n128, npairs, 3900, 1000, 351));
+    consider(TileShape::kPair256, est(t2 * n256, npairs, 3800, 2900, 375, 256, 2, &q));
+    if (n128) consider(TileShape::kPair128, est(t2 * n128, npairs, 3900, 1000, 351, 128, 2, &q));
   }
   return best;
 }
@@ -64,16 +89,17 @@ cudaError_t launch_out(const GemmArgs& a) {
       return launch_cfg<256, false, false, kX, OutT>(a);
     } else {
       // gated layers always take 256-wide tiles: a tile's gate and up rows meet in one epilogue
-      switch (token_major_shape(a)) {
+      GemmArgs b = a;
+      switch (token_major_shape(a, &b.parts)) {
         case TileShape::kPair256:
-          return a.gated ? launch_cfg<256, false, true, kX, OutT, false, true>(a)
-                         : launch_cfg<256, false, false, kX, OutT, false, true>(a);
+          return b.gated ? launch_cfg<256, false, true, kX, OutT, false, true>(b)
+                         : launch_cfg<256, false, false, kX, OutT, false, true>(b);
         case TileShape::kPair128:
-          return launch_cfg<128, false, false, kX, OutT, false, true>(a);
+          return launch_cfg<128, false, false, kX, OutT, false, true>(b);
         case TileShape::kSingle128:
-          return launch_cfg<128, false, false, kX, OutT>(a);
+          return launch_cfg<128, false, false, kX, OutT>(b);
         default:
-          return a.gated ? launch_cfg<256, false, true, kX, OutT>(a) : launch_cfg<256, false, false, kX, OutT>(a);
+          return b.gated ? launch_cfg<256, false, true, kX, OutT>(b) : launch_cfg<256, false, false, kX, OutT>(b);
       }
     }
   }

@@ -114,6 +114,13 @@ struct Params {
   int M, N;      // N = weight rows of the layer (2H for a gated layer)
   int ldy;       // row length of y (N, or H for a gated layer)
   int splits;    // weight-major orientation: CTAs of a cluster splitting K (1 = no split)
+  // token-major, non-gated: each tile's k-blocks in `parts` work units (1 = whole tiles), each
+  // unit's FP32 partial in part_ws [tile][part][CTA of the pair][kBN / 4][kBM] (float4 elements);
+  // part_cnt [tile][CTA of the pair] counts the finished units (zero at launch; the tile's last
+  // unit adds the partials to its own, applies the epilogue and resets the count)
+  int parts;
+  float* part_ws;
+  int* part_cnt;
   float kconst;  // the zero-point constant of the accumulator: 64 K (int4 codes), 1024 K (int8)
   // per-group step scales (kGroup): the step's scales [ngroups], each group's code sums of the
   // activations [M][ngroups] and 8 x of the weights [N][ngroups], k-blocks per group, 64 x
@@ -411,6 +418,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   __shared__ int s_xs[kFused ? kBN : 1];        // fused: code sums of each token over this CTA's k-range
   __shared__ uint32_t s_tmem_base;
   __shared__ int s_epi_abort;  // set by an epilogue thread whose wait timed out
+  __shared__ int s_last;       // split of K: this unit was its tile's last to finish
   // per-column parameters of the current tile (non-swap): weight scale, code correction, bias
   __shared__ __align__(16) float s_ws[kSwap ? 1 : kBN];
   __shared__ __align__(16) float s_wc[kSwap ? 1 : kBN];
@@ -423,6 +431,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   const int tiles_b = (p.rows_b + kBN - 1) / kBN;
   const int ntiles = tiles_a * tiles_b;
   const int nkb_all = p.K / kBK;
+  const int parts = p.parts;
+  const int nunits = ntiles * parts;
   // split-K (weight-major orientation): the `splits` CTAs of a cluster share one tile, CTA r
   // taking k-blocks [kb0, kb1); without a split every CTA runs whole tiles persistently
   const int splits = kSwap ? p.splits : 1;
@@ -438,6 +448,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
   // across the role loops they would cost a register in every role)
 #define QVLA_UNIT0 (blockIdx.x / static_cast<unsigned>(udiv))
 #define QVLA_NUNITS (gridDim.x / static_cast<unsigned>(udiv))
+  // work unit u: tile u / parts, k-blocks [ka, kz) of this CTA's range (all of it when parts = 1)
+  auto unit_range = [&](int u, int& tile, int& ka, int& kz) {
+    tile = u / parts;
+    const int part = u - tile * parts;
+    ka = kb0 + (kb1 - kb0) * part / parts;
+    kz = kb0 + (kb1 - kb0) * (part + 1) / parts;
+  };
   uint8_t* const raw = smem + C::kStages * C::kStage;  // staging ring after the expanded stages
 
   if (threadIdx.x == 0) {
@@ -559,9 +576,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       griddep_wait();
       int it = 0;
       bool ok = !hold;
-      for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS) {
+      for (int u = QVLA_UNIT0; u < nunits && ok; u += QVLA_NUNITS) {
+        int tile, ka, kz;
+        unit_range(u, tile, ka, kz);
         const int ta = tile % tiles_a, tb = tile / tiles_a;
-        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+        for (int kb = ka; kb < kz; ++kb, ++it) {
           const int s = it % C::kStages;
           const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
           if (it >= pre) {
@@ -644,8 +663,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
     }
     int it = 0;
     bool ok = true;
-    for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS) {
-      for (int kb = kb0; kb < kb1; ++kb, ++it) {
+    for (int u = QVLA_UNIT0; u < nunits && ok; u += QVLA_NUNITS) {
+      int tile, ka, kz;
+      unit_range(u, tile, ka, kz);
+      for (int kb = ka; kb < kz; ++kb, ++it) {
         const int s = it % C::kStages;
         const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
         if (!mbar_wait(smem_u32(&bar_raw_full[s]), ph)) { ok = false; break; }
@@ -679,13 +700,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       constexpr uint32_t kIdesc = idesc_e4m3_f32(2 * kBM, kBN);
       int it = 0, tile_iter = 0;
       bool ok = true;
-      for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS, ++tile_iter) {
+      for (int u = QVLA_UNIT0; u < nunits && ok; u += QVLA_NUNITS, ++tile_iter) {
+        int tile, ka, kz;
+        unit_range(u, tile, ka, kz);
+        (void)tile;
         const int buf = tile_iter & 1;
         const uint32_t aph = static_cast<uint32_t>(tile_iter >> 1) & 1u;
         if (!mbar_wait(smem_u32(&bar_tempty[buf]), aph ^ 1u)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d = tmem_base + static_cast<uint32_t>(buf * kBN);
-        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+        for (int kb = ka; kb < kz; ++kb, ++it) {
           const int s = it % C::kStages;
           const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
           if (!mbar_wait(smem_u32(&bar_full[s]), ph)) { ok = false; break; }
@@ -695,7 +719,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
 #pragma unroll
           for (int kk = 0; kk < kBK / 32; ++kk)
             mma_e4m3_pair(d, smem_desc_sw128(sa + kk * 32), smem_desc_sw128(sb + kk * 32), kIdesc,
-                          (kb != kb0 || kk != 0) ? 1u : 0u);
+                          (kb != ka || kk != 0) ? 1u : 0u);
           mma_commit_pair(smem_u32(&bar_empty[s]), 3);  // both CTAs' stage s is free
         }
         if (!ok) break;
@@ -708,12 +732,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       // the leader (the converters themselves arrive locally)
       int it = 0;
       bool ok = true;
-      for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS)
-        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+      for (int u = QVLA_UNIT0; u < nunits && ok; u += QVLA_NUNITS) {
+        int tile, ka, kz;
+        unit_range(u, tile, ka, kz);
+        (void)tile;
+        for (int kb = ka; kb < kz; ++kb, ++it) {
           const int s = it % C::kStages;
           if (!mbar_wait(smem_u32(&bar_full[s]), static_cast<uint32_t>(it / C::kStages) & 1u)) { ok = false; break; }
           mbar_arrive_peer(mapa_shared(smem_u32(&bar_full[s]), 0));
         }
+      }
     } else if (kPair) {
       // the other lanes of a pair's MMA warp have no role
     } else if (lane == 0 && kGroup) {
@@ -750,7 +778,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
       constexpr uint32_t kIdesc = idesc_e4m3_f32(kBM, kBN);
       int it = 0, tile_iter = 0;
       bool ok = true;
-      for (int tile = QVLA_UNIT0; tile < ntiles && ok; tile += QVLA_NUNITS, ++tile_iter) {
+      for (int u = QVLA_UNIT0; u < nunits && ok; u += QVLA_NUNITS, ++tile_iter) {
+        int tile, ka, kz;
+        unit_range(u, tile, ka, kz);
+        (void)tile;
         const int buf = tile_iter & 1;
         const uint32_t aph = static_cast<uint32_t>(tile_iter >> 1) & 1u;
         if (!mbar_wait(smem_u32(&bar_tempty[buf]), aph ^ 1u)) { ok = false; break; }
@@ -759,7 +790,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
           if (!mbar_wait_cluster(smem_u32(&bar_xready), 0)) { ok = false; break; }
         }
         const uint32_t d = tmem_base + static_cast<uint32_t>(buf * kBN);
-        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+        for (int kb = ka; kb < kz; ++kb, ++it) {
           const int s = it % C::kStages;
           const uint32_t ph = static_cast<uint32_t>(it / C::kStages) & 1u;
           if (!mbar_wait(smem_u32(&bar_full[s]), ph)) { ok = false; break; }
@@ -774,7 +805,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
 #pragma unroll
             for (int kk = 0; kk < kBK / 32; ++kk) {
               mma_e4m3(d, smem_desc_sw128(pa + kk * 32), smem_desc_sw128(pb + kk * 32), kIdesc,
-                       (kb != kb0 || pl != 0 || kk != 0) ? 1u : 0u);
+                       (kb != ka || pl != 0 || kk != 0) ? 1u : 0u);
             }
           }
           mma_commit(smem_u32(&bar_empty[s]));
@@ -919,7 +950,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
         if (!ok) continue;
       }
     } else
-    for (int tile = QVLA_UNIT0; tile < ntiles; tile += QVLA_NUNITS, ++tile_iter) {
+    for (int u = QVLA_UNIT0; u < nunits; u += QVLA_NUNITS, ++tile_iter) {
+      int tile, ka, kz;
+      unit_range(u, tile, ka, kz);
+      (void)ka;
+      (void)kz;
+      const int part = u - tile * parts;
       const int ta = tile % tiles_a, tb = tile / tiles_a;
       const int buf = tile_iter & 1;
       const uint32_t aph = static_cast<uint32_t>(tile_iter >> 1) & 1u;
@@ -952,12 +988,61 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
         const float xs = mok ? p.xscale[m] : 0.0f;
         const float cm = mok ? 8.0f * static_cast<float>(p.xsum[m]) + k64 : 0.0f;
         OutT* yrow = reinterpret_cast<OutT*>(p.y) + static_cast<size_t>(mok ? m : 0) * p.ldy;
+        // split of K (parts > 1): this unit's partial goes to its slot, and the tile's last unit
+        // to finish adds the other units' slots to its own accumulator (exact: every partial is a
+        // non-negative integer multiple of the same power of two, and so is their sum, below 2^24
+        // of them).  A slot holds float4 (row r, columns 4j .. 4j+3) at j * kBM + r, so the 32
+        // rows of a warp move 512 contiguous bytes per access.  On a CTA pair each CTA has slots
+        // and a count of its own 128 rows: slot (tile, part, CTA rank), count (tile, CTA rank).
+        constexpr int kHalves = kPair ? 2 : 1;
+        constexpr int kSlot4 = kBM * kBN / 4;
+        const int half = static_cast<int>(prank);
+        float4* const slot4 = parts > 1 ? reinterpret_cast<float4*>(p.part_ws) + static_cast<size_t>((tile * parts + part) * kHalves + half) * kSlot4 + et : nullptr;
+        bool last = parts == 1;
+        if (parts > 1) {
 #pragma unroll 1
-        for (int c0 = 0; c0 < kBN; c0 += 32) {
+          for (int c0 = 0; c0 < kBN; c0 += 32) {
+            uint32_t r[32];
+            __syncwarp();
+            tmem_ld32(taddr + c0, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 32; i += 4)
+              __stcg(slot4 + ((c0 + i) / 4) * kBM, make_float4(__uint_as_float(r[i]), __uint_as_float(r[i + 1]),
+                                                                __uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])));
+          }
+          // the slot is written (every row: the barrier, then the counting thread's fence) before
+          // the unit is counted, and the last unit reads the slots after its fence
+          epi_sync();
+          if (et == 0) {
+            __threadfence();
+            s_last = atomicAdd(p.part_cnt + tile * kHalves + half, 1) == parts - 1;
+          }
+          epi_sync();
+          last = s_last != 0;
+          if (last) __threadfence();
+        }
+#pragma unroll 1
+        for (int c0 = 0; c0 < kBN && last; c0 += 32) {
           uint32_t r[32];
           __syncwarp();
           tmem_ld32(taddr + c0, r);
           tmem_ld_wait();
+#pragma unroll 1
+          for (int q = 0; q < parts; ++q) {
+            if (q == part) continue;
+            const float4* const o4 = slot4 + static_cast<ptrdiff_t>(q - part) * kHalves * kSlot4 + (c0 / 4) * kBM;
+            float4 v[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) v[j] = __ldcg(o4 + j * kBM);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              r[4 * j] = __float_as_uint(__uint_as_float(r[4 * j]) + v[j].x);
+              r[4 * j + 1] = __float_as_uint(__uint_as_float(r[4 * j + 1]) + v[j].y);
+              r[4 * j + 2] = __float_as_uint(__uint_as_float(r[4 * j + 2]) + v[j].z);
+              r[4 * j + 3] = __float_as_uint(__uint_as_float(r[4 * j + 3]) + v[j].w);
+            }
+          }
           const int n0 = tb * kBN + c0;
           if (mok && n0 < p.N) {
             const int nvalid = min(32, p.N - n0);
@@ -989,6 +1074,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_w4a4_kernel(const __grid_con
             }
           }
         }
+        if (parts > 1 && last && et == 0) p.part_cnt[tile * kHalves + half] = 0;  // ready for the next launch
       } else if constexpr (!kSwap && kGated) {
         // Gated MLP: tile columns [0, kBN/2) are the gate rows of hidden units
         // j0 .. j0 + kBN/2 - 1 and columns [kBN/2, kBN) the up rows of the same units.
@@ -1347,6 +1433,9 @@ cudaError_t launch_fused_cfg(const GemmArgs& a) {
   p.N = a.N;
   p.ldy = a.N;
   p.splits = splits;
+  p.parts = 1;
+  p.part_ws = nullptr;
+  p.part_cnt = nullptr;
   p.x = a.x;
   p.log_b = a.log_b;
   p.inv_sqrt_b = a.inv_sqrt_b;
@@ -1429,12 +1518,27 @@ cudaError_t launch_cfg(const GemmArgs& a) {
     }
   }
   p.splits = splits;
+  // token-major tiles of a non-gated layer: each tile's k-blocks in a.parts work units over the
+  // persistent CTAs (or pairs), partials in the caller's workspace, when it has room for them
+  p.parts = 1;
+  p.part_ws = nullptr;
+  p.part_cnt = nullptr;
+  if constexpr (!kSwap && !kGated && !kGroup && kX <= 1) {
+    const long halves = kPair ? 2 : 1;
+    if (a.parts > 1 && a.part_ws != nullptr && a.part_cnt != nullptr && p.K / kBK >= a.parts &&
+        static_cast<size_t>(tiles) * halves * a.parts * kBM * kBN <= a.part_ws_floats && tiles * halves <= a.part_cnt_n) {
+      p.parts = a.parts;
+      p.part_ws = a.part_ws;
+      p.part_cnt = a.part_cnt;
+    }
+  }
   attr[1].val.clusterDim.x = static_cast<unsigned>(kPair ? 2 : splits);
   if (kPair) {
-    const int pairs = a.num_sms / 2;
-    cfg.gridDim = dim3(2 * (tiles < pairs ? tiles : pairs));
+    const int pairs = a.num_sms / 2, units = tiles * p.parts;
+    cfg.gridDim = dim3(2 * (units < pairs ? units : pairs));
   } else {
-    cfg.gridDim = dim3(splits > 1 ? tiles * splits : (tiles < a.num_sms ? tiles : a.num_sms));
+    const int units = tiles * p.parts;
+    cfg.gridDim = dim3(splits > 1 ? tiles * splits : (units < a.num_sms ? units : a.num_sms));
   }
   cfg.attrs = attr;
   cfg.numAttrs = (kPair || splits > 1) ? 2 : 1;  // a cluster launch for pairs and when K is split

@@ -29,6 +29,8 @@ struct RotQuantArgs {
                            //   holds whole Hadamard blocks and >= 128 channels): step_scale
                            //   then points at the step's [K >> gshift] entries, absmax too
   int32_t* xgsum = nullptr;  // device [M][K >> gshift] per-group code sums, or null
+  int32_t* zero = nullptr;   // device ints set to 0 once x has been waited for (the next GEMM's
+  int zero_n = 0;            //   work-unit counters), or null
   cudaStream_t stream;
 };
 bool rotate_quant_supported(int log_b);
@@ -85,6 +87,15 @@ struct GemmArgs {
   int xdt = 0;
   int log_b = 0;
   float inv_sqrt_b = 1.0f;
+  // token-major tiles of a non-gated layer may split their k-blocks into `parts` work units
+  // when the tiles leave SMs idle: the units' FP32 partials go to part_ws (part_ws_floats
+  // floats) and part_cnt (part_cnt_n ints, zero at launch; the GEMM leaves them zero) counts
+  // each tile's finished units.  Null: no split.  `parts` is set by the tile-shape choice.
+  int parts = 1;
+  float* part_ws = nullptr;
+  size_t part_ws_floats = 0;
+  int* part_cnt = nullptr;
+  int part_cnt_n = 0;
   int num_sms;
   cudaStream_t stream;
 };

@@ -141,7 +141,8 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
                                                              const float* __restrict__ step_scale,
                                                              uint8_t* __restrict__ xq, float* __restrict__ xscale,
                                                              int32_t* __restrict__ xsum, float* __restrict__ absmax_out,
-                                                             int out_mode, int gshift, int32_t* __restrict__ xgsum) {
+                                                             int out_mode, int gshift, int32_t* __restrict__ xgsum,
+                                                             int32_t* __restrict__ zero, int zero_n) {
   constexpr float kQ = kA8 ? 127.0f : 7.0f;
   constexpr float kBand = kA8 ? kTieBand8 : kTieBand;
   constexpr int kP = (kEpt == 128) ? 7 : 6;  // log2(kEpt)
@@ -181,6 +182,8 @@ __global__ void __launch_bounds__(256) rotate_quant_kernel(const T* __restrict__
 
   griddep_wait();  // x comes from the previous kernel, which may still read xq / xscale / xsum
   griddep_launch_dependents();
+  if (zero != nullptr && blockIdx.x == 0)  // the next GEMM's work-unit counters (its previous use is over)
+    for (int i = tid; i < zero_n; i += blockDim.x) zero[i] = 0;
   float2 v[kN];
   if (active) {
     const T* src = x + static_cast<size_t>(m) * K + static_cast<size_t>(j) * kEpt;
@@ -516,7 +519,7 @@ cudaError_t launch_t(const RotQuantArgs& a) {
   cfg.numAttrs = 1;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, reinterpret_cast<const T*>(a.x), a.M, a.K, a.inv_sqrt_b, a.step_scale,
                                      a.xq, a.xscale, a.xsum, a.mode == 2 ? a.absmax : nullptr, a.out_mode,
-                                     a.gshift, a.xgsum);
+                                     a.gshift, a.xgsum, a.zero, a.zero_n);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

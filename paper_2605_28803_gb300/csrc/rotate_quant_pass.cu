@@ -35,6 +35,8 @@ struct RqpParams {
   float* xscale;            // [M]
   int32_t* xsum;            // [M] or null
   const float* step_scale;  // per-step mode: the step's scale
+  int32_t* zero;            // ints set to 0 once x has been waited for, or null
+  int zero_n;
   int M, K, C, P, log_b;
   float inv_sqrt_b;
 };
@@ -65,6 +67,8 @@ __global__ void __launch_bounds__(kRqpThreads) rotate_quant_pass_kernel(RqpParam
   }
   griddep_wait();  // x comes from the previous kernel, which may still read xq / xscale / xsum
   griddep_launch_dependents();
+  if (p.zero != nullptr && blockIdx.x == 0)  // the next GEMM's work-unit counters
+    for (int i = threadIdx.x; i < p.zero_n; i += kRqpThreads) p.zero[i] = 0;
 
   float2 v[4];
   const bool holds = 8 * t < C;  // the thread holds channels 8 t .. 8 t + 7 of the pass
@@ -240,6 +244,8 @@ cudaError_t launch_rotate_quant_pass(const RotQuantArgs& a, bool* launched) {
   p.xscale = a.xscale;
   p.xsum = a.xsum;
   p.step_scale = a.step_scale;
+  p.zero = a.zero;
+  p.zero_n = a.zero_n;
   p.M = a.M;
   p.K = a.K;
   p.C = C;

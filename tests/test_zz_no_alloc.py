@@ -78,7 +78,9 @@ def test_noalloc_rejects_more_rows_than_its_scratch_holds():
 def test_noalloc_counts_the_online_rotation_in_its_scratch():
     # A layer with an online x.P.BlockDiag(U_b) keeps x' in the scratch as well: 2000 rows of
     # K = 2048 fit without it (operand bytes and sums) but not with 2000 x 2048 bf16 values more.
-    K, N, M = 2048, 256, 2000
+    # (N = 2560: 16 x 10 tiles of 128 x 256, enough for every SM, so the workspace has no
+    # split-of-K part.)
+    K, N, M = 2048, 2560, 2000
     case = W.sweep_linear(16, K, N, seed=24, xdtype="bf16", ydtype="bf16")
     layer = _layer(case, "bf16", "bf16")
     assert Q.qvla_linear_workspace_bytes(layer, M) <= Q.NOALLOC_SCRATCH_BYTES
