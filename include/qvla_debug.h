@@ -1,7 +1,8 @@
 /*
  * libqvla test hooks.  They have no counterpart in the paper: they exist so that the tests can
  * make one of the kernels' bounded waits run out (the failure path of QVLA_ERR_TIMEOUT in
- * qvla.h) without a GPU fault, a trap or a hang.  Off by default; not for production use.
+ * qvla.h) without a GPU fault, a trap or a hang, and read the GEMM's host-side launch plan on a
+ * machine without a GPU.  Off by default; not for production use.
  */
 #ifndef QVLA_DEBUG_H
 #define QVLA_DEBUG_H
@@ -27,6 +28,20 @@ extern "C" {
  * Synchronises the device first; affects every later launch on the current device until called
  * again. */
 qvla_status qvla_debug_set_hooks(unsigned long long wait_limit_ns, int hold_gemm_loads);
+
+/* The launch plan that qvla_w4a4_linear's GEMM (Sec. 4.2, Eq. 7) takes for M > 128 tokens of an
+ * M x K -> N layer on a device of num_sms SMs: the host-side choice of tile shape and split of K,
+ * computed without touching a device.
+ *   N          the layer's weight rows (2H for a gated layer)
+ *   gated      nonzero: a gated gate/up layer (qvla_layer_create_gated)
+ *   split_room nonzero: the workspace has the room qvla_linear_workspace_bytes counts for the
+ *              split of K; 0: the linear runs in a workspace of the required parts only
+ *   shape      out: 0 single CTAs with 128 x 128 tiles, 1 single CTAs with 128 x 256, 2 CTA pairs
+ *              with 256 x 128, 3 CTA pairs with 256 x 256 (tokens x weight rows)
+ *   parts      out: work units per tile; 1 = whole tiles
+ * QVLA_ERR_INVALID_ARG for null outputs, M <= 128 (those batches run weight-major), K not a
+ * positive multiple of 128, N not a positive multiple of 16 (256 when gated), num_sms < 2. */
+qvla_status qvla_debug_gemm_plan(int M, int K, int N, int gated, int num_sms, int split_room, int* shape, int* parts);
 
 #ifdef __cplusplus
 }

@@ -652,14 +652,17 @@ constexpr int kMaxParts = 4;  // work units per tile of the GEMM's split of K
 // The GEMM's split of K: a non-gated token-major layer (M > 128) whose 128 x 256 tiles leave SMs
 // idle may split; room for kMaxParts FP32 partials of every output (rows and weight rows padded to
 // 256) and a count for each 128 x 128 tile covers every tile shape it can take.
-bool may_split(const qvla_layer* L, int M) {
-  if (M <= 128 || L->gated) return false;
-  return static_cast<long>((M + 127) / 128) * ((L->N + 255) / 256) < num_sms(L->device);
+bool may_split_mn(int M, int N, bool gated, int sms) {
+  if (M <= 128 || gated) return false;
+  return static_cast<long>((M + 127) / 128) * ((N + 255) / 256) < sms;
 }
-size_t split_floats(const qvla_layer* L, int M) {
-  return static_cast<size_t>((M + 255) / 256) * 256 * ((L->N + 255) / 256) * 256 * kMaxParts;
+size_t split_floats_mn(int M, int N) {
+  return static_cast<size_t>((M + 255) / 256) * 256 * ((N + 255) / 256) * 256 * kMaxParts;
 }
-int split_counts(const qvla_layer* L, int M) { return ((M + 127) / 128) * ((L->N + 127) / 128); }
+int split_counts_mn(int M, int N) { return ((M + 127) / 128) * ((N + 127) / 128); }
+bool may_split(const qvla_layer* L, int M) { return may_split_mn(M, L->N, L->gated != 0, num_sms(L->device)); }
+size_t split_floats(const qvla_layer* L, int M) { return split_floats_mn(M, L->N); }
+int split_counts(const qvla_layer* L, int M) { return split_counts_mn(M, L->N); }
 size_t workspace_parts(const qvla_layer* L, int M) {
   if (!may_split(L, M)) return 0;
   return round256(split_floats(L, M) * 4) + round256(static_cast<size_t>(split_counts(L, M)) * 4);
@@ -1000,6 +1003,33 @@ qvla_status qvla_debug_set_hooks(unsigned long long wait_limit_ns, int hold_gemm
   QVLA_CUDA(qvla::set_debug_hooks_fused(limit, hold), "test hooks (fused)");
   QVLA_CUDA(qvla::set_debug_hooks_gemv(limit, hold), "test hooks (gemv)");
   QVLA_CUDA(qvla::set_debug_hooks_rqp(limit, hold), "test hooks (rotate-quantise)");
+  return QVLA_OK;
+}
+
+qvla_status qvla_debug_gemm_plan(int M, int K, int N, int gated, int sms, int split_room, int* shape, int* parts) {
+  g_last_error.clear();
+  if (!shape || !parts) return fail(QVLA_ERR_INVALID_ARG, "shape and parts must not be NULL");
+  if (M <= 128) return fail(QVLA_ERR_INVALID_ARG, "M=%d: up to 128 rows run weight-major, not token-major", M);
+  if (K <= 0 || K % 128 != 0) return fail(QVLA_ERR_INVALID_ARG, "K=%d must be a positive multiple of 128", K);
+  if (N <= 0 || N % 16 != 0 || (gated && N % 256 != 0))
+    return fail(QVLA_ERR_INVALID_ARG, "N=%d must be a positive multiple of 16 (of 256 when gated)", N);
+  if (sms < 2) return fail(QVLA_ERR_INVALID_ARG, "num_sms=%d must be at least 2", sms);
+  qvla::GemmArgs a = {};
+  a.x_bytes = 1;
+  a.M = M;
+  a.N = N;
+  a.K = K;
+  a.gated = gated ? 1 : 0;
+  a.num_sms = sms;
+  static float no_floats;  // stand-ins for the workspace: the plan reads only whether it is there
+  static int no_counts;
+  if (split_room && may_split_mn(M, N, gated != 0, sms)) {
+    a.part_ws = &no_floats;
+    a.part_ws_floats = split_floats_mn(M, N);
+    a.part_cnt = &no_counts;
+    a.part_cnt_n = split_counts_mn(M, N);
+  }
+  *shape = qvla::token_major_plan(a, parts);
   return QVLA_OK;
 }
 

@@ -112,6 +112,8 @@ cudaError_t launch_out(const GemmArgs& a) {
 
 }  // namespace
 
+int token_major_plan(const GemmArgs& a, int* parts) { return static_cast<int>(token_major_shape(a, parts)); }
+
 cudaError_t launch_gemm_w4a4(const GemmArgs& a) {
   if (a.M == 0) return cudaSuccess;
   {  // one to four tokens: the weight stream decides, so the CUDA-core GEMV takes it

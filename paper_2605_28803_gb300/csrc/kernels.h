@@ -100,6 +100,11 @@ struct GemmArgs {
   cudaStream_t stream;
 };
 cudaError_t launch_gemm_w4a4(const GemmArgs& a);
+// The token-major launch plan of launch_gemm_w4a4 for int4 operand-byte activations and M > 128
+// (host logic only; a's device pointers are not read): the tile shape (0 single CTAs 128 x 128,
+// 1 single CTAs 128 x 256, 2 CTA pairs 256 x 128, 3 CTA pairs 256 x 256) and *parts, the work
+// units per tile (1 = whole tiles).
+int token_major_plan(const GemmArgs& a, int* parts);
 
 // The one-launch linear for a small batch with a per-step scale (gemm_fused.cu): the weight-major
 // split-K GEMM whose CTAs rotate and quantise the activations themselves.  *launched is false

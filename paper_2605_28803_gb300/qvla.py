@@ -56,6 +56,7 @@ SIGNATURES = {
     "qvla_gemm_w4a8": (_I, [_P, _P, _P, _I, _P, _P, _P, _S, _P]),
     "qvla_check_device": (_I, [_P]),
     "qvla_debug_set_hooks": (_I, [ctypes.c_ulonglong, _I]),
+    "qvla_debug_gemm_plan": (_I, [_I, _I, _I, _I, _I, _I, _P, _P]),
 }
 
 
@@ -301,3 +302,16 @@ def qvla_debug_set_hooks(wait_limit_ns: int = 0, hold_gemm_loads: bool = False) 
     """Test hooks (include/qvla_debug.h): the device wait limit (0 = default) and whether GEMM
     load warps hold back every copy."""
     _check(_lib.qvla_debug_set_hooks(int(wait_limit_ns), 1 if hold_gemm_loads else 0))
+
+
+GEMM_SHAPES = ("single 128x128", "single 128x256", "pair 256x128", "pair 256x256")
+
+
+def qvla_debug_gemm_plan(M: int, K: int, N: int, gated: bool = False, num_sms: int = 152,
+                         split_room: bool = True) -> tuple[str, int]:
+    """The token-major GEMM's launch plan (include/qvla_debug.h): (tile shape, work units per
+    tile) for M > 128 tokens of an M x K -> N layer (N weight rows, 2H when gated).  Host only."""
+    shape, parts = ctypes.c_int(-1), ctypes.c_int(0)
+    _check(_lib.qvla_debug_gemm_plan(M, K, N, 1 if gated else 0, num_sms, 1 if split_room else 0,
+                                     ctypes.addressof(shape), ctypes.addressof(parts)))
+    return GEMM_SHAPES[shape.value], parts.value
