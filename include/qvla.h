@@ -294,10 +294,14 @@ qvla_status qvla_w4a4_linear_fused(const qvla_layer* layer, const void* x, int M
  * qvla_linear_quantize rotates and quantises x into `workspace` (as qvla_rotate_quantize, step
  * as there); qvla_linear_gemm then runs the integer GEMM and epilogue on it (as qvla_gemm_w4a4).
  * The workspace contents in between are internal to the library: the codes as tensor-core
- * operand bytes, the scales and the code sums.  Same workspace rules as qvla_w4a4_linear. */
+ * operand bytes, the scales and the code sums, which the GEMM only reads, and the counters of
+ * the GEMM's split of K, which qvla_linear_quantize zeroes and the GEMM leaves zero (it uses the
+ * split's room as scratch).  So qvla_linear_gemm must follow a qvla_linear_quantize of the same
+ * layer, M and workspace; it may run again on the same codes.  Same workspace rules as
+ * qvla_w4a4_linear. */
 qvla_status qvla_linear_quantize(const qvla_layer* layer, const void* x, int M, int step, void* workspace,
                                  size_t workspace_bytes, void* stream);
-qvla_status qvla_linear_gemm(const qvla_layer* layer, const void* workspace, size_t workspace_bytes, int M, void* y,
+qvla_status qvla_linear_gemm(const qvla_layer* layer, void* workspace, size_t workspace_bytes, int M, void* y,
                              void* stream);
 
 /* Allocation-free variant of qvla_w4a4_linear.  The paper has no counterpart: this entry

@@ -741,7 +741,7 @@ qvla_status qvla_linear_quantize(const qvla_layer* L, const void* x, int M, int 
                    nullptr, w.parts.cnt, w.parts.n);
 }
 
-qvla_status qvla_linear_gemm(const qvla_layer* L, const void* workspace, size_t workspace_bytes, int M, void* y,
+qvla_status qvla_linear_gemm(const qvla_layer* L, void* workspace, size_t workspace_bytes, int M, void* y,
                              void* stream) {
   g_last_error.clear();
   if (!L) return fail(QVLA_ERR_INVALID_ARG, "layer must not be NULL");
@@ -750,7 +750,7 @@ qvla_status qvla_linear_gemm(const qvla_layer* L, const void* workspace, size_t 
   if (!y) return fail(QVLA_ERR_INVALID_ARG, "y must not be NULL");
   if (!aligned16(y)) return fail(QVLA_ERR_INVALID_ARG, "y must be 16-byte aligned");
   LinearWorkspace w;
-  if (qvla_status s = carve_workspace(L, M, const_cast<void*>(workspace), workspace_bytes, &w)) return s;
+  if (qvla_status s = carve_workspace(L, M, workspace, workspace_bytes, &w)) return s;
   return launch_gemm(L, w.xb, 1, w.xscale, w.xsum, M, y, nullptr, stream, nullptr, nullptr, &w.parts);
 }
 
